@@ -1,0 +1,7 @@
+"""CPU float64 oracle of the GRPO scoring + loss + backward path.
+
+Test infrastructure: only the tests, ``__graft_entry__.smoke()`` and ``bench.py``'s
+``cpu_baseline`` leg use it. It shares no code with the CUDA path.
+"""
+from .grpo_oracle import (SEQ_MEAN, TOKEN_MEAN, aggregate, group_advantages, grpo_step,  # noqa: F401
+                          logit_grads, param_grads, score_tokens, token_objective, valid_counts)

@@ -1,0 +1,220 @@
+"""Plain CPU float64 oracle of one GRPO update's token-scoring, loss and backward path.
+
+TEST INFRASTRUCTURE. Only the test suite, ``__graft_entry__.smoke()`` and the ``cpu_baseline``
+leg of ``bench.py`` may import or run this module. It shares no code with the CUDA path and
+imports nothing from the package: callers hand it plain numpy arrays.
+
+What it computes (arxiv 2510.17158):
+
+* Eq. 1 (Sec. 2.1, "Fine-tuning LMs with RL") is the GRPO objective
+  ``L = E_{x~pi}[-w(x) log pi(x|c)] + beta KL(pi || pi_ref)``, where ``w(x)`` is the reward of
+  ``x`` normalised within its group of K completions (Sec. 2.1; Alg. 1, "normalize within each
+  group").
+* Sec. 6.1 ("GRPO Adaptations") keeps "the traditional GRPO policy" of DeepSeekMath, i.e. the
+  per-token probability ratio with a clipped surrogate; Alg. 1 computes the KL to a frozen
+  reference and takes a gradient step on L.
+* ``log pi(x|c)`` is the sum over the completion's sampled tokens of the log-softmax of the
+  LM-head logits ``z_t = W h_t`` at the sampled token.
+
+Readings of points the paper leaves open (each one is a documented choice):
+
+* advantage = z-score within the group, ``(r - mean) / (std + std_eps)``; std unbiased by
+  default (population on request); a group of one, or whose rewards are all equal, gets 0;
+* ratio ``rho = exp(logp - old)``; surrogate ``min(rho A, clip(rho, 1-eps_lo, 1+eps_hi) A)``;
+* KL per sampled token with the non-negative estimator ``e^delta - delta - 1``,
+  ``delta = ref - logp``;
+* per-token loss ``l = -surr + beta kl``; aggregation "seq_mean" ``(1/S) sum_i (1/n_i) sum_t l``
+  (default; a sequence with no scored token adds 0 and still counts in S) or "token_mean"
+  ``sum l / sum n``; masked tokens (padding, tool-result text) are not scored;
+* the subgradient of the clipped surrogate takes the unclipped branch when it is active with
+  inclusive boundaries: active iff (A >= 0 and rho <= 1+eps_hi) or (A < 0 and rho >= 1-eps_lo);
+* argmax ties go to the lowest vocabulary index; entropy is in nats.
+
+Every input is converted exactly to float64 (bf16 and fp32 values are exactly representable).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+SEQ_MEAN = "seq_mean"
+TOKEN_MEAN = "token_mean"
+
+
+def _f64(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+def valid_counts(mask):
+    """n_i = number of scored tokens of completion i (Eq. 1 takes its expectation over sampled
+    completion tokens; tool-result text appended inside a completion (Sec. 5) is not sampled
+    from the policy and is masked out)."""
+    m = np.asarray(mask)
+    return (m != 0).sum(axis=1).astype(np.int64)
+
+
+def group_advantages(rewards, group_offsets, std_mode="unbiased", std_eps=1e-4):
+    """w(x_k) of Eq. 1: the reward of completion k normalised within its group (Sec. 2.1;
+    Alg. 1, "normalize within each group to get advantages").
+
+    ``group_offsets[g] .. group_offsets[g+1]`` are the completions of prompt g (contiguous).
+    """
+    r = _f64(rewards)
+    go = np.asarray(group_offsets, dtype=np.int64)
+    adv = np.zeros_like(r)
+    for g in range(len(go) - 1):
+        lo, hi = int(go[g]), int(go[g + 1])
+        G = hi - lo
+        if G <= 1:
+            continue
+        rg = r[lo:hi]
+        if np.all(np.asarray(rewards)[lo:hi] == np.asarray(rewards)[lo]):
+            continue                      # degenerate group: no relative signal, advantage 0
+        mu = rg.sum() / G
+        dof = G - 1 if std_mode == "unbiased" else G
+        sigma = np.sqrt(((rg - mu) ** 2).sum() / dof)
+        adv[lo:hi] = (rg - mu) / (sigma + std_eps)
+    return adv
+
+
+def score_tokens(h, W, y):
+    """Per-token scoring of Eq. 1's log pi(x|c): for each row h_t and sampled token y_t,
+    z_t = W h_t over the whole vocabulary, lse_t = log sum_v exp(z_tv), logp_t = z_t[y_t] - lse_t,
+    entropy_t = -sum_v p_tv log p_tv = lse_t - sum_v p_tv z_tv, argmax_t = first v with the
+    largest z_tv.
+
+    h: [n, d]; W: [V, d]; y: [n] ints in [0, V).
+    """
+    h = _f64(h)
+    W = _f64(W)
+    y = np.asarray(y, dtype=np.int64)
+    n = h.shape[0]
+    Z = h @ W.T                                   # logits, [n, V]
+    m = Z.max(axis=1)
+    lse = m + np.log(np.exp(Z - m[:, None]).sum(axis=1))
+    logp = Z[np.arange(n), y] - lse
+    P = np.exp(Z - lse[:, None])
+    entropy = lse - (P * Z).sum(axis=1)
+    rows = np.arange(n)
+    argmax = Z.argmax(axis=1)                     # numpy returns the first maximal index
+    # runner-up (tie diagnostics only): the best logit once the argmax entry is removed
+    Z[rows, argmax] = -np.inf
+    second = Z.argmax(axis=1)
+    Z[rows, argmax] = m
+    gap = m - Z[rows, second] if Z.shape[1] > 1 else np.full(n, np.inf)
+    return {"logp": logp, "lse": lse, "entropy": entropy, "argmax": argmax, "top_gap": gap,
+            "second": second}
+
+
+def token_objective(logp, old, ref, adv_tok, eps_low, eps_high, beta):
+    """Per-token GRPO terms (Sec. 6.1 clipped-ratio surrogate; Eq. 1 KL term with the
+    per-token estimator) and their derivative with respect to logp.
+
+    Returns rho, surr, kl, ell = -surr + beta*kl, and dell = d ell / d logp.
+    """
+    logp, old, ref, A = _f64(logp), _f64(old), _f64(ref), _f64(adv_tok)
+    rho = np.exp(logp - old)
+    unclipped = rho * A
+    clipped = np.clip(rho, 1.0 - eps_low, 1.0 + eps_high) * A
+    surr = np.minimum(unclipped, clipped)
+    delta = ref - logp
+    kl = np.exp(delta) - delta - 1.0
+    ell = -surr + beta * kl
+    active = ((A >= 0) & (rho <= 1.0 + eps_high)) | ((A < 0) & (rho >= 1.0 - eps_low))
+    dsurr = np.where(active, A * rho, 0.0)        # d(rho A)/dlogp = A rho where unclipped is taken
+    dkl = 1.0 - np.exp(delta)                     # d(e^delta - delta - 1)/dlogp
+    dell = -dsurr + beta * dkl
+    return {"rho": rho, "surr": surr, "kl": kl, "ell": ell, "dell": dell, "active": active}
+
+
+def aggregate(ell, dell, seq_of_token, counts, num_seqs, agg=SEQ_MEAN, norm=None):
+    """Loss L over the scored tokens and g_t = dL/dlogp_t (Eq. 1's expectation). Also returns
+    sum_t |w_t l_t|, the magnitude against which L's rounding error is measured.
+
+    seq_mean:   L = (1/S) sum_i (1/n_i) sum_t l_t        (S = norm or num_seqs)
+    token_mean: L = sum_t l_t / N                          (N = norm or sum_i n_i)
+    """
+    ell, dell = _f64(ell), _f64(dell)
+    seq = np.asarray(seq_of_token, dtype=np.int64)
+    n = np.asarray(counts, dtype=np.float64)
+    if agg == SEQ_MEAN:
+        S = float(norm) if norm else float(num_seqs)
+        w_tok = 1.0 / (S * n[seq])
+    elif agg == TOKEN_MEAN:
+        N = float(norm) if norm else float(n.sum())
+        w_tok = np.full(ell.shape, 1.0 / N)
+    else:
+        raise ValueError(agg)
+    L = float((w_tok * ell).sum())
+    g = w_tok * dell
+    mass = float(np.abs(w_tok * ell).sum())      # sum of |terms|: the scale of L's rounding
+    return L, g, mass
+
+
+def logit_grads(h, W, y, lse, g):
+    """dL/dz_t = g_t (onehot(y_t) - softmax(z_t)) for each scored token (chain rule through
+    logp_t = z_t[y_t] - lse_t)."""
+    h, W, lse, g = _f64(h), _f64(W), _f64(lse), _f64(g)
+    y = np.asarray(y, dtype=np.int64)
+    Z = h @ W.T
+    P = np.exp(Z - lse[:, None])
+    onehot = np.zeros_like(P)
+    onehot[np.arange(len(y)), y] = 1.0
+    return g[:, None] * (onehot - P)
+
+
+def param_grads(h, W, y, lse, g, vocab_rows=None):
+    """dL/dh_t = W^T dz_t and dL/dW = sum_t dz_t h_t^T (Alg. 1's gradient step on L, for the
+    LM head and its input). ``vocab_rows`` restricts dW to a subset of rows (exact, since a row
+    of dW needs only its own column of dz)."""
+    dZ = logit_grads(h, W, y, lse, g)
+    dH = dZ @ _f64(W)
+    if vocab_rows is None:
+        dW = dZ.T @ _f64(h)
+    else:
+        dW = dZ[:, vocab_rows].T @ _f64(h)
+    return dH, dW
+
+
+def grpo_step(H, W, tokens, mask, rewards, group_offsets, old, ref, eps_low=0.2, eps_high=0.2,
+              beta=0.04, agg=SEQ_MEAN, std_mode="unbiased", std_eps=1e-4, norm=None,
+              adv=None, vocab_rows=None, with_grads=True):
+    """The whole path on a padded batch: H [S,T,d], W [V,d], tokens/mask/old/ref [S,T],
+    rewards [S]. Returns per-position outputs ([S,T], zeros at unscored positions, argmax -1),
+    per-sequence counts and advantages, the loss, g, dH [S,T,d] and dW [V,d] (or its rows)."""
+    H = _f64(H)
+    S, T, d = H.shape
+    mask = np.asarray(mask)
+    counts = valid_counts(mask)
+    if adv is None:
+        adv = group_advantages(rewards, group_offsets, std_mode, std_eps)
+    idx = np.argwhere(mask != 0)
+    si, ti = idx[:, 0], idx[:, 1]
+    h = H[si, ti]
+    y = np.asarray(tokens)[si, ti]
+    sc = score_tokens(h, W, y)
+    out = {"counts": counts, "adv": adv}
+    for k in ("logp", "lse", "entropy"):
+        a = np.zeros((S, T))
+        a[si, ti] = sc[k]
+        out[k] = a
+    am = np.full((S, T), -1, dtype=np.int64)
+    am[si, ti] = sc["argmax"]
+    out["argmax"] = am
+    gap = np.full((S, T), np.inf)
+    gap[si, ti] = sc["top_gap"]
+    out["top_gap"] = gap
+    tob = token_objective(sc["logp"], _f64(old)[si, ti], _f64(ref)[si, ti], adv[si],
+                          eps_low, eps_high, beta)
+    L, g_tok, mass = aggregate(tob["ell"], tob["dell"], si, counts, S, agg, norm)
+    out["loss"] = L
+    out["loss_abs_mass"] = mass
+    g = np.zeros((S, T))
+    g[si, ti] = g_tok
+    out["g"] = g
+    if with_grads:
+        dHv, dW = param_grads(h, W, y, sc["lse"], g_tok, vocab_rows)
+        dH = np.zeros((S, T, d))
+        dH[si, ti] = dHv
+        out["dH"] = dH
+        out["dW"] = dW
+    return out
