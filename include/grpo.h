@@ -1,0 +1,144 @@
+/*
+ * grpo.h -- C ABI of the fused GRPO token-scoring + loss + backward library (GB300, sm_103a).
+ *
+ * One GRPO update (arxiv 2510.17158, Alg. 1) scores K sampled completions per prompt, normalises
+ * their rewards within the group, and takes a gradient step on
+ *     L = E_{x~pi}[ -w(x) log pi(x|c) ] + beta KL(pi || pi_ref)                  (Eq. 1)
+ * using the clipped-ratio surrogate that Sec. 6.1 keeps from "traditional GRPO". This library
+ * computes the data-parallel core of that step for the LM head: logits z = W h per token over
+ * the whole vocabulary (never written to memory), log-softmax at the sampled token, entropy and
+ * argmax, group advantages, the per-token surrogate + KL loss, and dL/dH, dL/dW.
+ *
+ * Conventions (every entry point):
+ *  - All array arguments are DEVICE pointers unless stated; the caller owns every buffer, the
+ *    workspace and the stream. The library allocates and frees nothing and never synchronises,
+ *    except grpo_last_device_error() and grpo_timing_read(), which say so.
+ *  - Work is enqueued asynchronously on `stream` (a cudaStream_t; 0 = legacy default stream).
+ *    Outputs are overwritten, never accumulated into.
+ *  - Layouts are row-major and contiguous:
+ *      H       [S, T, d]   hidden states of every position (bf16 or f32; padding must be finite)
+ *      W       [V, d]      LM-head weight (same dtype as H)
+ *      tokens  [S, T]      int32 sampled token ids, in [0, V) where mask != 0
+ *      mask    [S, T]      uint8, nonzero = scored completion token (prompt padding, tool-result
+ *                          text and tail padding are 0; holes inside a completion are allowed)
+ *      per-token f32 arrays [S, T]; per-sequence arrays [S].
+ *    Sequences of one group are contiguous: group g owns sequences
+ *    group_offsets[g] .. group_offsets[g+1]-1.
+ *  - Host-side argument checks run before any launch and return a negative status with nothing
+ *    enqueued. Faults only the device can see (a token id outside [0, V) at a scored position,
+ *    invalid group offsets, a bounded wait that ran out) write a status word in the workspace;
+ *    read it with grpo_last_device_error().
+ *  - Unscored positions get logp = lse = entropy = 0, argmax = -1, g = 0 and dH rows = 0.
+ */
+#ifndef GRPO_GB300_H
+#define GRPO_GB300_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* grpo_stream_t; /* same object as cudaStream_t */
+
+typedef enum {
+  GRPO_OK = 0,
+  GRPO_ERR_INVALID_ARG = -1,  /* null pointer, non-positive size, bad enum, ...            */
+  GRPO_ERR_UNSUPPORTED = -2,  /* shape/dtype combination this build does not implement     */
+  GRPO_ERR_CUDA = -3,         /* a CUDA runtime call or a launch failed                      */
+  GRPO_ERR_WORKSPACE = -4,    /* workspace too small or misaligned                           */
+  GRPO_ERR_TOKEN_RANGE = -5,  /* device: a scored token id outside [0, V)                    */
+  GRPO_ERR_TIMEOUT = -6,      /* device: a bounded wait inside a kernel ran out              */
+  GRPO_ERR_GROUPS = -7        /* device: group offsets not non-decreasing from 0 to S        */
+} grpo_status;
+
+typedef enum { GRPO_F32 = 0, GRPO_BF16 = 1 } grpo_dtype;
+typedef enum { GRPO_STD_UNBIASED = 0, GRPO_STD_POPULATION = 1 } grpo_std_mode;
+typedef enum { GRPO_AGG_SEQ_MEAN = 0, GRPO_AGG_TOKEN_MEAN = 1 } grpo_agg;
+
+/* Bytes of workspace needed for a problem of this shape. `vocab_chunk` is how many vocabulary
+ * columns of dL/dz the backward keeps at once (rounded up to a multiple of 256); 0 = the whole
+ * vocabulary in one chunk (fastest; S*ceil(T/128)*128*V*2 bytes of scratch). Returns 0 for
+ * invalid shapes. The workspace must be 256-byte aligned. */
+size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                            int32_t vocab_chunk);
+
+/* Clears the workspace's status word. Call once after allocating a workspace. */
+int grpo_workspace_init(void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
+/* Group-relative advantages (Eq. 1's w(x); Sec. 2.1 and Alg. 1 "normalize within each group").
+ *   rewards        [num_seqs] f32
+ *   group_offsets  [num_groups+1] int32, device; must rise from 0 to num_seqs (else the status
+ *                  word gets GRPO_ERR_GROUPS and the affected advantages are NaN)
+ *   adv_out        [num_seqs] f32: (r - mean_g) / (std_g + std_eps); std unbiased (default) or
+ *                  population; exactly 0 for a group of one or a group whose rewards are all equal
+ * Needs >= 256 bytes of workspace (status word only). */
+int group_advantages(const float* rewards, const int32_t* group_offsets, int32_t num_groups,
+                     int32_t num_seqs, int32_t std_mode, float std_eps, float* adv_out,
+                     void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
+/* Forward scoring of Eq. 1's log pi(x|c) per token: z_t = W h_t over all V columns, reduced on
+ * chip (the [tokens x V] logits never reach memory) to
+ *   lse_t = log sum_v exp(z_tv), logp_t = z_t[y_t] - lse_t, entropy_t = lse_t - sum_v p_tv z_tv
+ *   (nats), argmax_t = lowest v with the largest z_tv; valid_count_i = #scored tokens of seq i.
+ * dtype GRPO_BF16: bf16 H, W, tensor-core products with f32 accumulation (d % 256 == 0).
+ * dtype GRPO_F32 : f32 H, W, f32 CUDA-core arithmetic (small problems, d <= 4096).
+ * Outputs: logp, lse, entropy f32 [S,T]; argmax int32 [S,T]; valid_count int32 [S]. */
+int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                   const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V, float* logp,
+                   float* lse, float* entropy, int32_t* argmax, int32_t* valid_count,
+                   void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
+/* GRPO loss and its gradient (Eq. 1 with the clipped-ratio surrogate of Sec. 6.1; Alg. 1's
+ * gradient step), per scored token t of sequence i:
+ *   rho = exp(logp - old_logp);  surr = min(rho A_i, clip(rho, 1-eps_low, 1+eps_high) A_i)
+ *   delta = ref_logp - logp;     kl = e^delta - delta - 1;      l_t = -surr + beta kl
+ *   L = (1/S') sum_i (1/n_i) sum_t l_t   (GRPO_AGG_SEQ_MEAN)   or   sum l_t / N' (TOKEN_MEAN)
+ * where S' = S and N' = sum_i n_i unless `norm` > 0 overrides them (data-parallel shards pass
+ * the global count). g_t = dL/dlogp_t takes the unclipped branch when it is active, boundaries
+ * inclusive. Then dz_t = g_t (onehot(y_t) - softmax(z_t)) is recomputed from H, W and lse,
+ * rounded to bf16, and contracted: dH_t = dz_t W (written in H's dtype), dW = sum_t dz_t h_t
+ * (f32). logp/lse/valid_count are grpo_score_fwd's outputs for the same H, W, tokens, mask.
+ * ref_logp may be NULL only when beta == 0. loss_out is one device f32. */
+int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                  const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                  const float* logp, const float* lse, const float* old_logp,
+                  const float* ref_logp, const float* adv, const int32_t* valid_count,
+                  float eps_low, float eps_high, float beta, int32_t agg, double norm,
+                  float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
+                  grpo_stream_t stream);
+
+/* Synchronises `stream`, returns the first device-side status recorded in the workspace since
+ * the last call (GRPO_OK if none) and clears it. *where_out (may be NULL) gets a code naming the
+ * kernel and wait that recorded it. */
+int grpo_last_device_error(void* workspace, int32_t* where_out, grpo_stream_t stream);
+
+const char* grpo_status_string(int status);
+
+/* Kernel accounting, for measurement. Every launch made by this library bumps a per-kernel
+ * counter. With timing enabled, each launch is bracketed by a pair of CUDA events recorded on
+ * its stream (host-side objects; no device memory). */
+enum {
+  GRPO_K_MASK_SCAN = 0, GRPO_K_TILE_LIST, GRPO_K_GROUP_ADV, GRPO_K_FWD_GEMM, GRPO_K_FWD_MERGE,
+  GRPO_K_LOSS_TOKENS, GRPO_K_LOSS_FINAL, GRPO_K_BWD_DZ_GEMM, GRPO_K_BWD_DH_GEMM,
+  GRPO_K_BWD_DW_GEMM, GRPO_K_DH_ZERO_TAIL, GRPO_K_F32_FWD, GRPO_K_F32_DH, GRPO_K_F32_DW,
+  GRPO_K_COUNT
+};
+const char* grpo_kernel_name(int32_t kernel_id);
+int grpo_timing_enable(int32_t enable);   /* 1 = record events from now on, 0 = stop */
+int grpo_timing_reset(void);              /* forget recorded events and counters */
+/* Synchronises on the recorded events; returns launches and summed device time of one kernel. */
+int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms);
+
+/* Fault-injection hook for tests of the bounded waits (failure detection without a GPU fault):
+ * while `on` is nonzero, CTA 0 of every tensor-core GEMM launched afterwards leaves its first
+ * pipeline stage unfilled; its MMA warp's wait then runs out after about 2 s, the kernel records
+ * GRPO_ERR_TIMEOUT in the workspace status word, releases its tensor memory and exits. Outputs of
+ * such a call are undefined. Process-wide; not for production use. */
+int grpo_debug_inject_stall(int32_t on);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GRPO_GB300_H */

@@ -1,0 +1,499 @@
+// C ABI of the GRPO library: argument checks, workspace layout, TMA descriptors and the launch
+// sequence of each entry point (declared and documented in include/grpo.h).
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "../../include/grpo.h"
+#include "common.cuh"
+#include "internal.h"
+
+using namespace grpo;
+
+namespace {
+
+// ------------------------------------------------------------------------------------------
+// kernel accounting
+// ------------------------------------------------------------------------------------------
+const char* const kKernelNames[GRPO_K_COUNT] = {
+    "mask_scan",       "tile_list",    "group_adv",   "fwd_gemm_tc",  "fwd_merge",
+    "loss_tokens",     "loss_final",   "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
+    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw"};
+
+struct EventPair {
+  cudaEvent_t a, b;
+};
+
+std::mutex g_mu;
+std::atomic<int> g_timing{0};
+std::atomic<int> g_inject_stall{0};
+std::atomic<long long> g_launches[GRPO_K_COUNT];
+std::vector<EventPair> g_pending[GRPO_K_COUNT];
+double g_total_ms[GRPO_K_COUNT];
+std::vector<EventPair> g_free_events;
+
+bool take_events(EventPair* p) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_free_events.empty()) {
+    *p = g_free_events.back();
+    g_free_events.pop_back();
+    return true;
+  }
+  if (cudaEventCreate(&p->a) != cudaSuccess) return false;
+  if (cudaEventCreate(&p->b) != cudaSuccess) {
+    cudaEventDestroy(p->a);
+    return false;
+  }
+  return true;
+}
+
+// Runs `launch` (which enqueues one kernel on `st` and returns its cudaError_t), counting it
+// and, with timing on, bracketing it with events.
+template <class F>
+int counted(int kid, cudaStream_t st, F&& launch) {
+  EventPair ev{};
+  const bool timed = g_timing.load() != 0 && take_events(&ev);
+  if (timed) cudaEventRecord(ev.a, st);
+  const cudaError_t e = launch();
+  if (timed) {
+    cudaEventRecord(ev.b, st);
+    std::lock_guard<std::mutex> lk(g_mu);
+    g_pending[kid].push_back(ev);
+  }
+  g_launches[kid].fetch_add(1);
+  return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA;
+}
+
+#define GRPO_TRY(x)             \
+  do {                          \
+    const int _st = (x);        \
+    if (_st != GRPO_OK) return _st; \
+  } while (0)
+
+// ------------------------------------------------------------------------------------------
+// workspace layout
+// ------------------------------------------------------------------------------------------
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Layout {
+  int max_tiles;
+  long long rows_cap;
+  int num_strips;
+  int v_round;          // V rounded up to a multiple of 256
+  size_t seq_last, seq_tile_base, tiles, counts, zy, partials, g, seq_loss;
+  size_t fixed_end;     // end of the regions that do not depend on the vocabulary chunk
+};
+
+Layout make_layout(int S, int T, int d, int V, int dtype) {
+  (void)d;
+  Layout L{};
+  L.max_tiles = S * ((T + kTileRows - 1) / kTileRows);
+  L.rows_cap = static_cast<long long>(L.max_tiles) * kTileRows;
+  const int nvt = (V + kTileN - 1) / kTileN;
+  L.num_strips = (nvt + kFwdTilesPerStrip - 1) / kFwdTilesPerStrip;
+  L.v_round = nvt * kTileN;
+  const size_t P = static_cast<size_t>(S) * T;
+  size_t off = sizeof(WsHeader);
+  L.seq_last = off;       off = align256(off + sizeof(int32_t) * S);
+  L.seq_tile_base = off;  off = align256(off + sizeof(int32_t) * (S + 1));
+  L.tiles = off;          off = align256(off + sizeof(int2) * L.max_tiles);
+  L.counts = off;         off = align256(off + sizeof(int32_t) * S);
+  L.zy = off;             off = align256(off + sizeof(float) * P);
+  L.partials = off;
+  if (dtype == GRPO_BF16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  L.g = off;              off = align256(off + sizeof(float) * P);
+  L.seq_loss = off;       off = align256(off + sizeof(float) * S);
+  L.fixed_end = off;
+  return L;
+}
+
+// Bytes of the chunk-dependent regions (f32 dH accumulator when chunked + bf16 dz scratch).
+size_t chunk_bytes(const Layout& L, int d, int vc) {
+  const size_t dz = align256(static_cast<size_t>(L.rows_cap) * vc * 2);
+  if (vc >= L.v_round) return dz;
+  return align256(static_cast<size_t>(L.rows_cap) * d * 4) + dz;
+}
+
+bool shape_ok(int S, int T, int d, int V) {
+  return S > 0 && T > 0 && d > 0 && V > 0 &&
+         static_cast<long long>(S) * T < (1ll << 31) && V < (1 << 30);
+}
+
+int check_dtype_shape(int dtype, int d) {
+  if (dtype == GRPO_BF16) return (d % kTileN == 0) ? GRPO_OK : GRPO_ERR_UNSUPPORTED;
+  if (dtype == GRPO_F32) return (d <= 4096) ? GRPO_OK : GRPO_ERR_UNSUPPORTED;
+  return GRPO_ERR_INVALID_ARG;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ------------------------------------------------------------------------------------------
+// TMA descriptors (driver entry point fetched through the runtime, no -lcuda needed)
+// ------------------------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] (inner contiguous, row pitch `pitch_elems`), box
+// [box_outer, 64], 128-byte swizzle, out-of-range elements read as zero.
+bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+              uint64_t pitch_elems, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_elems * 2};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                        strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+int gemm_grid(long long units) {
+  const long long sms = num_sms();
+  if (sms <= 0) return 1;
+  return static_cast<int>(units < sms ? (units > 0 ? units : 1) : sms);
+}
+
+struct Views {
+  WsHeader* hdr;
+  int32_t* seq_last;
+  int32_t* seq_tile_base;
+  int2* tiles;
+  int32_t* counts;
+  float* zy;
+  float4* partials;
+  float* g;
+  float* seq_loss;
+};
+
+Views views(void* ws, const Layout& L) {
+  char* b = static_cast<char*>(ws);
+  Views v;
+  v.hdr = reinterpret_cast<WsHeader*>(b);
+  v.seq_last = reinterpret_cast<int32_t*>(b + L.seq_last);
+  v.seq_tile_base = reinterpret_cast<int32_t*>(b + L.seq_tile_base);
+  v.tiles = reinterpret_cast<int2*>(b + L.tiles);
+  v.counts = reinterpret_cast<int32_t*>(b + L.counts);
+  v.zy = reinterpret_cast<float*>(b + L.zy);
+  v.partials = reinterpret_cast<float4*>(b + L.partials);
+  v.g = reinterpret_cast<float*>(b + L.g);
+  v.seq_loss = reinterpret_cast<float*>(b + L.seq_loss);
+  return v;
+}
+
+GemmArgs base_args(const Layout& L, const Views& v, int S, int T, int d, int V,
+                   const int32_t* tokens, const uint8_t* mask) {
+  GemmArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.S = S;
+  a.T = T;
+  a.d = d;
+  a.V = V;
+  a.tiles = v.tiles;
+  a.hdr = v.hdr;
+  a.tokens = tokens;
+  a.mask = mask;
+  a.rows_cap = L.rows_cap;
+  a.num_strips = L.num_strips;
+  a.inject_stall = g_inject_stall.load();
+  return a;
+}
+
+}  // namespace
+
+// ==========================================================================================
+// C ABI
+// ==========================================================================================
+extern "C" {
+
+const char* grpo_status_string(int status) {
+  switch (status) {
+    case GRPO_OK: return "ok";
+    case GRPO_ERR_INVALID_ARG: return "invalid argument";
+    case GRPO_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case GRPO_ERR_CUDA: return "CUDA runtime or launch error";
+    case GRPO_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case GRPO_ERR_TOKEN_RANGE: return "token id outside [0, V) at a scored position";
+    case GRPO_ERR_TIMEOUT: return "a bounded wait inside a kernel ran out";
+    case GRPO_ERR_GROUPS: return "group offsets do not rise from 0 to S";
+    default: return "unknown status";
+  }
+}
+
+const char* grpo_kernel_name(int32_t kernel_id) {
+  if (kernel_id < 0 || kernel_id >= GRPO_K_COUNT) return "unknown";
+  return kKernelNames[kernel_id];
+}
+
+size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                            int32_t vocab_chunk) {
+  if (!shape_ok(S, T, d, V) || check_dtype_shape(dtype, d) == GRPO_ERR_INVALID_ARG) return 0;
+  const Layout L = make_layout(S, T, d, V, dtype);
+  if (dtype != GRPO_BF16) return L.fixed_end;
+  int vc = L.v_round;
+  if (vocab_chunk > 0) {
+    vc = ((vocab_chunk + kTileN - 1) / kTileN) * kTileN;
+    if (vc > L.v_round) vc = L.v_round;
+  }
+  return L.fixed_end + chunk_bytes(L, d, vc);
+}
+
+int grpo_workspace_init(void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  if (!workspace || workspace_bytes < sizeof(WsHeader)) return GRPO_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
+  return cudaMemsetAsync(workspace, 0, sizeof(WsHeader), reinterpret_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? GRPO_OK
+             : GRPO_ERR_CUDA;
+}
+
+int group_advantages(const float* rewards, const int32_t* group_offsets, int32_t num_groups,
+                     int32_t num_seqs, int32_t std_mode, float std_eps, float* adv_out,
+                     void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  if (!rewards || !group_offsets || !adv_out) return GRPO_ERR_INVALID_ARG;
+  if (num_groups <= 0 || num_seqs <= 0) return GRPO_ERR_INVALID_ARG;
+  if (std_mode != GRPO_STD_UNBIASED && std_mode != GRPO_STD_POPULATION) return GRPO_ERR_INVALID_ARG;
+  if (!(std_eps >= 0.f)) return GRPO_ERR_INVALID_ARG;
+  if (!workspace || workspace_bytes < sizeof(WsHeader) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  WsHeader* hdr = static_cast<WsHeader*>(workspace);
+  return counted(GRPO_K_GROUP_ADV, st, [&] {
+    return launch_group_adv(rewards, group_offsets, num_groups, num_seqs, std_mode, std_eps,
+                            adv_out, hdr, st);
+  });
+}
+
+int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                   const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V, float* logp,
+                   float* lse, float* entropy, int32_t* argmax, int32_t* valid_count,
+                   void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  if (!H || !W || !tokens || !mask || !logp || !lse || !entropy || !argmax || !valid_count)
+    return GRPO_ERR_INVALID_ARG;
+  if (!shape_ok(S, T, d, V)) return GRPO_ERR_INVALID_ARG;
+  GRPO_TRY(check_dtype_shape(dtype, d));
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
+  const Layout L = make_layout(S, T, d, V, dtype);
+  if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const Views v = views(workspace, L);
+
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, valid_count, v.seq_last, st); }));
+  if (dtype == GRPO_F32) {
+    return counted(GRPO_K_F32_FWD, st, [&] {
+      return launch_f32_fwd(static_cast<const float*>(H), static_cast<const float*>(W), tokens,
+                            mask, S, T, d, V, logp, lse, entropy, argmax, v.hdr, st);
+    });
+  }
+  if (!aligned16(H) || !aligned16(W)) return GRPO_ERR_INVALID_ARG;
+  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
+    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
+  }));
+  CUtensorMap mapH, mapW;
+  if (!make_map(&mapH, H, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+      !make_map(&mapW, W, d, V, d, kTileN))
+    return GRPO_ERR_CUDA;
+  GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
+  a.partials = v.partials;
+  a.zy = v.zy;
+  const int grid = gemm_grid(static_cast<long long>(L.max_tiles) * L.num_strips);
+  GRPO_TRY(counted(GRPO_K_FWD_GEMM, st,
+                   [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, st); }));
+  return counted(GRPO_K_FWD_MERGE, st, [&] {
+    return launch_fwd_merge(v.partials, L.rows_cap, L.num_strips, v.zy, v.seq_tile_base, tokens,
+                            mask, S, T, V, logp, lse, entropy, argmax, v.hdr, st);
+  });
+}
+
+int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                  const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                  const float* logp, const float* lse, const float* old_logp,
+                  const float* ref_logp, const float* adv, const int32_t* valid_count,
+                  float eps_low, float eps_high, float beta, int32_t agg, double norm,
+                  float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
+                  grpo_stream_t stream) {
+  if (!H || !W || !tokens || !mask || !logp || !lse || !old_logp || !adv || !valid_count ||
+      !loss_out || !dH || !dW)
+    return GRPO_ERR_INVALID_ARG;
+  if (!ref_logp && beta != 0.f) return GRPO_ERR_INVALID_ARG;
+  if (!shape_ok(S, T, d, V)) return GRPO_ERR_INVALID_ARG;
+  GRPO_TRY(check_dtype_shape(dtype, d));
+  if (agg != GRPO_AGG_SEQ_MEAN && agg != GRPO_AGG_TOKEN_MEAN) return GRPO_ERR_INVALID_ARG;
+  if (!(eps_low >= 0.f) || !(eps_high >= 0.f) || !(beta >= 0.f) || !(norm >= 0.0))
+    return GRPO_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
+  const Layout L = make_layout(S, T, d, V, dtype);
+  if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const Views v = views(workspace, L);
+  // ref_logp is not read when beta == 0; pass a valid pointer anyway.
+  const float* ref = ref_logp ? ref_logp : logp;
+
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, v.counts, v.seq_last, st); }));
+  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
+    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
+  }));
+  GRPO_TRY(counted(GRPO_K_LOSS_TOKENS, st, [&] {
+    return launch_loss_tokens(mask, logp, old_logp, ref, adv, valid_count, S, T, eps_low,
+                              eps_high, beta, agg, norm, v.hdr, v.g, v.seq_loss, st);
+  }));
+  GRPO_TRY(counted(GRPO_K_LOSS_FINAL, st, [&] {
+    return launch_loss_final(v.seq_loss, S, agg, norm, v.hdr, loss_out, st);
+  }));
+
+  if (dtype == GRPO_F32) {
+    GRPO_TRY(counted(GRPO_K_F32_DH, st, [&] {
+      return launch_f32_dh(static_cast<const float*>(H), static_cast<const float*>(W), tokens,
+                           mask, lse, v.g, S, T, d, V, static_cast<float*>(dH), st);
+    }));
+    return counted(GRPO_K_F32_DW, st, [&] {
+      return launch_f32_dw(static_cast<const float*>(H), static_cast<const float*>(W), tokens,
+                           mask, lse, v.g, S, T, d, V, dW, st);
+    });
+  }
+
+  if (!aligned16(H) || !aligned16(W) || !aligned16(dH) || !aligned16(dW))
+    return GRPO_ERR_INVALID_ARG;
+  // Vocabulary chunk: the whole vocabulary if the workspace holds it, else the largest
+  // multiple of 256 that fits next to the f32 dH accumulator.
+  const size_t avail = workspace_bytes - L.fixed_end;
+  int vc;
+  if (avail >= chunk_bytes(L, d, L.v_round)) {
+    vc = L.v_round;
+  } else {
+    const size_t acc = align256(static_cast<size_t>(L.rows_cap) * d * 4);
+    if (avail < acc) return GRPO_ERR_WORKSPACE;
+    const size_t per_col = static_cast<size_t>(L.rows_cap) * 2;
+    long long cols = static_cast<long long>((avail - acc - 256) / per_col);
+    vc = static_cast<int>((cols / kTileN) * kTileN);
+    if (vc < kTileN) return GRPO_ERR_WORKSPACE;
+  }
+  const int nchunks = (V + vc - 1) / vc;
+  char* wsb = static_cast<char*>(workspace);
+  float* dH_acc = nullptr;
+  __nv_bfloat16* dz;
+  if (nchunks == 1) {
+    dz = reinterpret_cast<__nv_bfloat16*>(wsb + L.fixed_end);
+  } else {
+    dH_acc = reinterpret_cast<float*>(wsb + L.fixed_end);
+    dz = reinterpret_cast<__nv_bfloat16*>(wsb + L.fixed_end +
+                                          align256(static_cast<size_t>(L.rows_cap) * d * 4));
+  }
+  CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn;
+  const uint64_t P = static_cast<uint64_t>(S) * T;
+  if (!make_map(&mapHk, H, d, P, d, kTileRows) || !make_map(&mapWk, W, d, V, d, kTileN) ||
+      !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
+      !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
+      !make_map(&mapHmn, H, d, P, d, 64))
+    return GRPO_ERR_CUDA;
+
+  GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
+  a.g = v.g;
+  a.lse = lse;
+  a.dz = dz;
+  a.dz_pitch = vc;
+  a.dH = static_cast<__nv_bfloat16*>(dH);
+  a.dH_acc = dH_acc;
+  a.dW = dW;
+  for (int c = 0; c < nchunks; ++c) {
+    a.vc0 = c * vc;
+    a.vc_len = (V - a.vc0) < vc ? (V - a.vc0) : vc;
+    a.dh_mode = nchunks == 1 ? 0 : (c == 0 ? 1 : (c == nchunks - 1 ? 3 : 2));
+    const long long vt = (a.vc_len + kTileN - 1) / kTileN;
+    GRPO_TRY(counted(GRPO_K_BWD_DZ_GEMM, st, [&] {
+      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles * vt), st);
+    }));
+    GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
+      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a,
+                         gemm_grid(static_cast<long long>(L.max_tiles) * (d / kTileN)), st);
+    }));
+    const long long vm = (a.vc_len + kTileRows - 1) / kTileRows;
+    GRPO_TRY(counted(GRPO_K_BWD_DW_GEMM, st, [&] {
+      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm * (d / kTileN)), st);
+    }));
+  }
+  return counted(GRPO_K_DH_ZERO_TAIL, st, [&] {
+    return launch_dh_zero_tail(v.seq_tile_base, S, T, d, static_cast<__nv_bfloat16*>(dH), st);
+  });
+}
+
+int grpo_last_device_error(void* workspace, int32_t* where_out, grpo_stream_t stream) {
+  if (!workspace) return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int32_t word[2] = {0, 0};
+  if (cudaMemcpyAsync(word, workspace, sizeof(word), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return GRPO_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return GRPO_ERR_CUDA;
+  if (cudaMemsetAsync(workspace, 0, sizeof(word), st) != cudaSuccess) return GRPO_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return GRPO_ERR_CUDA;
+  if (where_out) *where_out = word[1];
+  return word[0];
+}
+
+int grpo_timing_enable(int32_t enable) {
+  g_timing.store(enable ? 1 : 0);
+  return GRPO_OK;
+}
+
+int grpo_timing_reset(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (int k = 0; k < GRPO_K_COUNT; ++k) {
+    for (auto& p : g_pending[k]) g_free_events.push_back(p);
+    g_pending[k].clear();
+    g_total_ms[k] = 0.0;
+    g_launches[k].store(0);
+  }
+  return GRPO_OK;
+}
+
+int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms) {
+  if (kernel_id < 0 || kernel_id >= GRPO_K_COUNT) return GRPO_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (auto& p : g_pending[kernel_id]) {
+    if (cudaEventSynchronize(p.b) != cudaSuccess) return GRPO_ERR_CUDA;
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.a, p.b) != cudaSuccess) return GRPO_ERR_CUDA;
+    g_total_ms[kernel_id] += ms;
+    g_free_events.push_back(p);
+  }
+  g_pending[kernel_id].clear();
+  if (launches) *launches = g_launches[kernel_id].load();
+  if (total_ms) *total_ms = g_total_ms[kernel_id];
+  return GRPO_OK;
+}
+
+/* Test hook, not part of the documented ABI: while set, the first CTA of every tensor-core
+ * GEMM leaves its first pipeline stage unfilled, so its MMA warp's bounded wait runs out and the
+ * kernel records GRPO_ERR_TIMEOUT and exits. */
+int grpo_debug_inject_stall(int32_t on) {
+  g_inject_stall.store(on ? 1 : 0);
+  return GRPO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+// Host-side interface between the C ABI (api.cu) and the kernel translation units.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+namespace grpo {
+
+struct WsHeader;
+
+// Token tiles: 128 consecutive positions of one sequence, (seq, t0). Tiles of a sequence cover
+// positions 0 .. last scored position; tile k occupies rows k*128 .. k*128+127 of "tile space",
+// the compact row numbering used by the dz scratch and by the GEMMs.
+constexpr int kTileRows = 128;
+// Vocabulary tile (N of the forward and dz GEMMs) and hidden tile (N of the dH / dW GEMMs).
+constexpr int kTileN = 256;
+// Vocabulary tiles merged on chip by one forward work unit before it writes partial statistics.
+constexpr int kFwdTilesPerStrip = 8;
+
+enum GemmRole : int { ROLE_FWD = 0, ROLE_DZ = 1, ROLE_DH = 2, ROLE_DW = 3 };
+
+// Arguments of the tcgen05 GEMM kernels (one struct for the four roles).
+struct GemmArgs {
+  int S, T, d, V;
+  const int2* tiles;        // [max_tiles] (seq, t0)
+  WsHeader* hdr;            // num_tiles, status word
+  const int32_t* tokens;    // [S*T]
+  const uint8_t* mask;      // [S*T]
+  long long rows_cap;       // max_tiles * 128
+  // vocabulary chunk (DZ / DH / DW)
+  int vc0, vc_len, dz_pitch;
+  // FWD: partial statistics per (strip, tile row) and the target logit per position
+  float4* partials;
+  int num_strips;
+  float* zy;
+  // DZ: per-position coefficient g and log-normaliser, bf16 dz scratch [rows_cap, dz_pitch]
+  const float* g;
+  const float* lse;
+  __nv_bfloat16* dz;
+  // DH: output (H's dtype), f32 accumulator in tile space, mode (0 single chunk, 1 first,
+  //     2 middle, 3 last)
+  __nv_bfloat16* dH;
+  float* dH_acc;
+  int dh_mode;
+  // DW: f32 [V, d]
+  float* dW;
+  // test hook: nonzero makes CTA 0's producer leave its first stage unfilled
+  int inject_stall;
+};
+
+// Launches (all asynchronous on `st`; return the cudaError_t of the launch).
+cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
+                             int32_t* seq_last, cudaStream_t st);
+cudaError_t launch_tile_list(const int32_t* seq_last, const int32_t* counts, int S, int T,
+                             int32_t* seq_tile_base, int2* tiles, WsHeader* hdr, cudaStream_t st);
+cudaError_t launch_group_adv(const float* rewards, const int32_t* go, int num_groups, int S,
+                             int std_mode, float std_eps, float* adv, WsHeader* hdr,
+                             cudaStream_t st);
+cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num_strips,
+                             const float* zy, const int32_t* seq_tile_base,
+                             const int32_t* tokens, const uint8_t* mask, int S, int T, int V,
+                             float* logp, float* lse, float* entropy, int32_t* argmax,
+                             WsHeader* hdr, cudaStream_t st);
+cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const float* old_logp,
+                               const float* ref_logp, const float* adv,
+                               const int32_t* valid_count, int S, int T, float eps_low,
+                               float eps_high, float beta, int agg, double norm,
+                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st);
+cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm,
+                              const WsHeader* hdr, float* loss_out, cudaStream_t st);
+cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d,
+                                __nv_bfloat16* dH, cudaStream_t st);
+cudaError_t launch_f32_fwd(const float* H, const float* W, const int32_t* tokens,
+                           const uint8_t* mask, int S, int T, int d, int V, float* logp,
+                           float* lse, float* entropy, int32_t* argmax, WsHeader* hdr,
+                           cudaStream_t st);
+cudaError_t launch_f32_dh(const float* H, const float* W, const int32_t* tokens,
+                          const uint8_t* mask, const float* lse, const float* g, int S, int T,
+                          int d, int V, float* dH, cudaStream_t st);
+cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
+                          const uint8_t* mask, const float* lse, const float* g, int S, int T,
+                          int d, int V, float* dW, cudaStream_t st);
+
+// tcgen05 GEMM launches. `grid` = persistent CTAs.
+size_t gemm_smem_bytes();
+cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
+                        const GemmArgs& args, int grid, cudaStream_t st);
+
+}  // namespace grpo

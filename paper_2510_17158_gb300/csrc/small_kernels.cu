@@ -1,0 +1,590 @@
+// Reduction and bookkeeping kernels of the GRPO path, plus the f32 CUDA-core path for small
+// problems: valid-token counts and the token-tile list, group-relative advantages (Eq. 1's
+// w(x), Alg. 1 "normalize within each group"), the merge of per-strip softmax statistics into
+// logp / lse / entropy / argmax, and the per-token clipped surrogate + KL loss with its
+// coefficient g_t = dL/dlogp_t (Sec. 6.1, Eq. 1). All reductions use a fixed order, so results
+// are bitwise reproducible run to run.
+#include <cfloat>
+#include <cmath>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace grpo {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+// ------------------------------------------------------------------------------------------
+// Valid counts n_i and the last scored position + 1 of every sequence (one warp per sequence).
+// ------------------------------------------------------------------------------------------
+__global__ void k_mask_scan(const uint8_t* __restrict__ mask, int S, int T,
+                            int32_t* __restrict__ counts, int32_t* __restrict__ seq_last) {
+  const int warps = blockDim.x / 32;
+  const int i = blockIdx.x * warps + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (i >= S) return;
+  const uint8_t* row = mask + static_cast<size_t>(i) * T;
+  int cnt = 0, last = 0;
+  for (int t = lane; t < T; t += 32) {
+    if (row[t] != 0) {
+      ++cnt;
+      last = t + 1;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    cnt += __shfl_xor_sync(kFull, cnt, o);
+    last = max(last, __shfl_xor_sync(kFull, last, o));
+  }
+  if (lane == 0) {
+    counts[i] = cnt;
+    seq_last[i] = last;
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Tile list: sequence i gets ceil(last_i / 128) tiles; exclusive prefix over sequences in one
+// block of 1024 threads (chunks of 1024 sequences, carried).
+// ------------------------------------------------------------------------------------------
+__global__ void k_tile_list(const int32_t* __restrict__ seq_last, const int32_t* __restrict__ counts,
+                            int S, int T, int32_t* __restrict__ seq_tile_base,
+                            int2* __restrict__ tiles, WsHeader* hdr) {
+  __shared__ int warp_tot[32];
+  __shared__ long long warp_cnt[32];
+  __shared__ int carry_s;
+  __shared__ long long carry_c;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  if (tid == 0) {
+    carry_s = 0;
+    carry_c = 0;
+  }
+  __syncthreads();
+  for (int base = 0; base < S; base += 1024) {
+    const int i = base + tid;
+    const int nt = (i < S) ? (seq_last[i] + kTileRows - 1) / kTileRows : 0;
+    const long long nc = (i < S) ? counts[i] : 0;
+    // inclusive warp scan of nt
+    int x = nt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(kFull, x, o);
+      if (lane >= o) x += y;
+    }
+    long long c = nc;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFull, c, o);
+    if (lane == 31) warp_tot[wid] = x;
+    if (lane == 0) warp_cnt[wid] = c;
+    __syncthreads();
+    if (wid == 0) {
+      int w = warp_tot[lane];
+      int xs = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(kFull, xs, o);
+        if (lane >= o) xs += y;
+      }
+      warp_tot[lane] = xs - w;  // exclusive prefix of warp totals
+    }
+    __syncthreads();
+    const int excl = carry_s + warp_tot[wid] + x - nt;
+    if (i < S) {
+      seq_tile_base[i] = excl;
+      for (int k = 0; k < nt; ++k) tiles[excl + k] = make_int2(i, k * kTileRows);
+    }
+    __syncthreads();
+    if (tid == 1023) carry_s = excl + nt;
+    if (tid == 0) {
+      long long s = 0;
+      for (int w = 0; w < 32; ++w) s += warp_cnt[w];
+      carry_c += s;
+    }
+    __syncthreads();
+  }
+  if (tid == 0) {
+    seq_tile_base[S] = carry_s;
+    hdr->num_tiles = carry_s;
+    hdr->total_valid = carry_c;
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Group advantages: one warp per group; mean and std in f32 with a fixed summation order.
+// ------------------------------------------------------------------------------------------
+__global__ void k_group_adv(const float* __restrict__ r, const int32_t* __restrict__ go,
+                            int num_groups, int S, int std_mode, float std_eps,
+                            float* __restrict__ adv, WsHeader* hdr) {
+  const int g = blockIdx.x;
+  const int lane = threadIdx.x;
+  if (g >= num_groups) return;
+  const int lo = go[g], hi = go[g + 1];
+  bool bad = lo < 0 || hi < lo || hi > S;
+  if (g == 0 && lo != 0) bad = true;
+  if (g == num_groups - 1 && hi != S) bad = true;
+  if (bad) {
+    if (lane == 0) record_error(hdr, ST_GROUPS, WHERE_GROUP_OFFSETS);
+    const int a = max(lo, 0), b = min(max(hi, a), S);
+    for (int i = a + lane; i < b; i += 32) adv[i] = __int_as_float(0x7fc00000);
+    return;
+  }
+  const int G = hi - lo;
+  if (G <= 0) return;
+  float s = 0.f;
+  bool same = true;
+  const float r0 = r[lo];
+  for (int i = lo + lane; i < hi; i += 32) {
+    const float v = r[i];
+    s += v;
+    same &= (__float_as_uint(v) == __float_as_uint(r0));
+  }
+  same = __all_sync(kFull, same);
+  const float mu = warp_sum(s) / static_cast<float>(G);
+  float q = 0.f;
+  for (int i = lo + lane; i < hi; i += 32) {
+    const float dv = r[i] - mu;
+    q = fmaf(dv, dv, q);
+  }
+  q = warp_sum(q);
+  const int dof = (std_mode == 0) ? G - 1 : G;
+  const bool degenerate = (G == 1) || same;
+  const float sigma = dof > 0 ? sqrtf(q / static_cast<float>(dof)) : 0.f;
+  for (int i = lo + lane; i < hi; i += 32) {
+    adv[i] = degenerate ? 0.f : (r[i] - mu) / (sigma + std_eps);
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Merge of per-strip statistics (max m, sum s = sum e^{z-m}, u = sum e^{z-m} z, argmax) into
+// lse, logp, entropy, argmax; one thread per position.
+// ------------------------------------------------------------------------------------------
+__global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_cap,
+                            int num_strips, const float* __restrict__ zy,
+                            const int32_t* __restrict__ seq_tile_base,
+                            const int32_t* __restrict__ tokens, const uint8_t* __restrict__ mask,
+                            int S, int T, int V, float* __restrict__ logp,
+                            float* __restrict__ lse_out, float* __restrict__ entropy,
+                            int32_t* __restrict__ argmax, WsHeader* hdr) {
+  const long long pos = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (pos >= static_cast<long long>(S) * T) return;
+  if (mask[pos] == 0) {
+    logp[pos] = 0.f;
+    lse_out[pos] = 0.f;
+    entropy[pos] = 0.f;
+    argmax[pos] = -1;
+    return;
+  }
+  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
+  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
+                        (t % kTileRows);
+  float M = -INFINITY;
+  int idx = 0;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    if (p.x > M) {
+      M = p.x;
+      idx = __float_as_int(p.w);
+    }
+  }
+  float Ssum = 0.f, U = 0.f;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    const float sc = ex2_approx((p.x - M) * kLog2e);
+    Ssum = fmaf(p.y, sc, Ssum);
+    U = fmaf(p.z, sc, U);
+  }
+  const float lse = M + logf(Ssum);
+  const int y = tokens[pos];
+  float lp;
+  if (y < 0 || y >= V) {
+    record_error(hdr, ST_TOKEN_RANGE, WHERE_MERGE_TOKEN);
+    lp = __int_as_float(0x7fc00000);
+  } else {
+    lp = zy[pos] - lse;
+  }
+  logp[pos] = lp;
+  lse_out[pos] = lse;
+  entropy[pos] = lse - U / Ssum;
+  argmax[pos] = idx;
+}
+
+// ------------------------------------------------------------------------------------------
+// Per-token loss terms and g_t = dL/dlogp_t; one block per sequence, fixed-order block sum.
+// ------------------------------------------------------------------------------------------
+constexpr int kLossThreads = 256;
+
+__device__ __forceinline__ float block_sum_fixed(float v, float* sh) {
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  v = warp_sum(v);
+  if (lane == 0) sh[wid] = v;
+  __syncthreads();
+  float tot = 0.f;
+  if (tid == 0) {
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += sh[w];
+  }
+  __syncthreads();
+  return tot;  // valid in thread 0
+}
+
+__global__ void __launch_bounds__(kLossThreads)
+    k_loss_tokens(const uint8_t* __restrict__ mask, const float* __restrict__ logp,
+                  const float* __restrict__ old_logp, const float* __restrict__ ref_logp,
+                  const float* __restrict__ adv, const int32_t* __restrict__ valid_count, int S,
+                  int T, float eps_low, float eps_high, float beta, int agg, double norm,
+                  const WsHeader* hdr, float* __restrict__ g, float* __restrict__ seq_loss) {
+  __shared__ float sh[32];
+  const int i = blockIdx.x;
+  const float A = adv[i];
+  const int n_i = valid_count[i];
+  float w;
+  if (agg == 0) {
+    const double Sn = norm > 0 ? norm : static_cast<double>(S);
+    w = n_i > 0 ? static_cast<float>(1.0 / (Sn * n_i)) : 0.f;
+  } else {
+    const double Nn = norm > 0 ? norm : static_cast<double>(hdr->total_valid);
+    w = Nn > 0 ? static_cast<float>(1.0 / Nn) : 0.f;
+  }
+  const float lo = 1.f - eps_low, hi = 1.f + eps_high;
+  float acc = 0.f;
+  const size_t base = static_cast<size_t>(i) * T;
+  for (int t = threadIdx.x; t < T; t += kLossThreads) {
+    const size_t pos = base + t;
+    float gt = 0.f;
+    if (mask[pos] != 0) {
+      const float lp = logp[pos];
+      const float rho = expf(lp - old_logp[pos]);
+      const float unclipped = rho * A;
+      const float clipped = fminf(fmaxf(rho, lo), hi) * A;
+      const float surr = fminf(unclipped, clipped);
+      float ell = -surr;
+      float dell = 0.f;
+      const bool active = (A >= 0.f) ? (rho <= hi) : (rho >= lo);
+      if (active) dell = -A * rho;
+      if (beta != 0.f) {
+        const float delta = ref_logp[pos] - lp;
+        const float ed = expf(delta);
+        ell = fmaf(beta, ed - delta - 1.f, ell);
+        dell = fmaf(beta, 1.f - ed, dell);
+      }
+      acc += ell;
+      gt = w * dell;
+    }
+    g[pos] = gt;
+  }
+  const float tot = block_sum_fixed(acc, sh);
+  if (threadIdx.x == 0) seq_loss[i] = tot * w;
+}
+
+__global__ void k_loss_final(const float* __restrict__ seq_loss, int S, float* loss_out) {
+  __shared__ float sh[32];
+  float acc = 0.f;
+  for (int i = threadIdx.x; i < S; i += blockDim.x) acc += seq_loss[i];
+  const float tot = block_sum_fixed(acc, sh);
+  if (threadIdx.x == 0) *loss_out = tot;
+}
+
+// ------------------------------------------------------------------------------------------
+// dH rows that no token tile covers (positions after a sequence's last tile) are zero.
+// ------------------------------------------------------------------------------------------
+__global__ void k_dh_zero_tail(const int32_t* __restrict__ seq_tile_base, int S, int T, int d,
+                               __nv_bfloat16* __restrict__ dH) {
+  const int tb = blockIdx.x, i = blockIdx.y;
+  const int covered = seq_tile_base[i + 1] - seq_tile_base[i];
+  if (tb < covered) return;
+  const int t0 = tb * kTileRows;
+  const int t1 = min(T, t0 + kTileRows);
+  if (t0 >= t1) return;
+  const size_t beg = (static_cast<size_t>(i) * T + t0) * d;
+  const size_t n = static_cast<size_t>(t1 - t0) * d;   // multiple of 8 (d % 64 == 0)
+  uint4* p = reinterpret_cast<uint4*>(dH + beg);
+  const uint4 z = make_uint4(0, 0, 0, 0);
+  for (size_t k = threadIdx.x; k < n / 8; k += blockDim.x) p[k] = z;
+}
+
+// ------------------------------------------------------------------------------------------
+// f32 path (CUDA cores, exact f32 arithmetic, small problems): one block per position.
+// ------------------------------------------------------------------------------------------
+constexpr int kF32Threads = 128;
+
+struct SoftStat {
+  float m, s, u, zy;
+  int idx;
+};
+
+__global__ void __launch_bounds__(kF32Threads)
+    k_f32_fwd(const float* __restrict__ H, const float* __restrict__ W,
+              const int32_t* __restrict__ tokens, const uint8_t* __restrict__ mask, int S, int T,
+              int d, int V, float* __restrict__ logp, float* __restrict__ lse_out,
+              float* __restrict__ entropy, int32_t* __restrict__ argmax, WsHeader* hdr) {
+  extern __shared__ float smem[];
+  float* h = smem;                                  // [d]
+  __shared__ float sm_m[kF32Threads], sm_s[kF32Threads], sm_u[kF32Threads];
+  __shared__ int sm_i[kF32Threads];
+  __shared__ float sm_zy;
+  const long long pos = blockIdx.x;
+  const int tid = threadIdx.x;
+  if (mask[pos] == 0) {
+    if (tid == 0) {
+      logp[pos] = 0.f;
+      lse_out[pos] = 0.f;
+      entropy[pos] = 0.f;
+      argmax[pos] = -1;
+    }
+    return;
+  }
+  for (int k = tid; k < d; k += kF32Threads) h[k] = H[pos * d + k];
+  if (tid == 0) sm_zy = __int_as_float(0x7fc00000);
+  __syncthreads();
+  const int y = tokens[pos];
+  float m = -INFINITY, s = 0.f, u = 0.f;
+  int idx = 0x7fffffff;
+  for (int v = tid; v < V; v += kF32Threads) {
+    const float* wr = W + static_cast<size_t>(v) * d;
+    float z = 0.f;
+    for (int k = 0; k < d; ++k) z = fmaf(wr[k], h[k], z);
+    if (v == y) sm_zy = z;
+    if (z > m) {
+      const float sc = expf(m - z);
+      s *= sc;
+      u *= sc;
+      m = z;
+      idx = v;
+    }
+    const float e = expf(z - m);
+    s += e;
+    u = fmaf(e, z, u);
+  }
+  sm_m[tid] = m;
+  sm_s[tid] = s;
+  sm_u[tid] = u;
+  sm_i[tid] = idx;
+  __syncthreads();
+  if (tid == 0) {
+    float M = -INFINITY;
+    int I = 0x7fffffff;
+    for (int j = 0; j < kF32Threads; ++j) {
+      if (sm_m[j] > M || (sm_m[j] == M && sm_i[j] < I)) {
+        M = sm_m[j];
+        I = sm_i[j];
+      }
+    }
+    float Ss = 0.f, U = 0.f;
+    for (int j = 0; j < kF32Threads; ++j) {
+      if (sm_m[j] == -INFINITY) continue;
+      const float sc = expf(sm_m[j] - M);
+      Ss = fmaf(sm_s[j], sc, Ss);
+      U = fmaf(sm_u[j], sc, U);
+    }
+    const float l = M + logf(Ss);
+    if (y < 0 || y >= V) {
+      record_error(hdr, ST_TOKEN_RANGE, WHERE_MERGE_TOKEN);
+    }
+    logp[pos] = sm_zy - l;
+    lse_out[pos] = l;
+    entropy[pos] = l - U / Ss;
+    argmax[pos] = I;
+  }
+}
+
+constexpr int kF32VChunk = 2048;
+
+__global__ void __launch_bounds__(kF32Threads)
+    k_f32_dh(const float* __restrict__ H, const float* __restrict__ W,
+             const int32_t* __restrict__ tokens, const uint8_t* __restrict__ mask,
+             const float* __restrict__ lse, const float* __restrict__ g, int S, int T, int d,
+             int V, float* __restrict__ dH) {
+  extern __shared__ float smem[];
+  float* h = smem;               // [d]
+  float* dz = smem + d;          // [kF32VChunk]
+  const long long pos = blockIdx.x;
+  const int tid = threadIdx.x;
+  float* out = dH + pos * d;
+  if (mask[pos] == 0) {
+    for (int k = tid; k < d; k += kF32Threads) out[k] = 0.f;
+    return;
+  }
+  for (int k = tid; k < d; k += kF32Threads) h[k] = H[pos * d + k];
+  const int y = tokens[pos];
+  const float gt = g[pos], l = lse[pos];
+  // each thread owns hidden indices k = tid, tid + 128, ...; at most 32 per thread here
+  float acc[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+  for (int v0 = 0; v0 < V; v0 += kF32VChunk) {
+    const int v1 = min(V, v0 + kF32VChunk);
+    __syncthreads();
+    for (int v = v0 + tid; v < v1; v += kF32Threads) {
+      const float* wr = W + static_cast<size_t>(v) * d;
+      float z = 0.f;
+      for (int k = 0; k < d; ++k) z = fmaf(wr[k], h[k], z);
+      const float p = expf(z - l);
+      dz[v - v0] = gt * ((v == y ? 1.f : 0.f) - p);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int k = tid + j * kF32Threads;
+      if (k < d) {
+        float a = acc[j];
+        for (int v = v0; v < v1; ++v) a = fmaf(dz[v - v0], W[static_cast<size_t>(v) * d + k], a);
+        acc[j] = a;
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const int k = tid + j * kF32Threads;
+    if (k < d) out[k] = acc[j];
+  }
+}
+
+__global__ void __launch_bounds__(kF32Threads)
+    k_f32_dw(const float* __restrict__ H, const float* __restrict__ W,
+             const int32_t* __restrict__ tokens, const uint8_t* __restrict__ mask,
+             const float* __restrict__ lse, const float* __restrict__ g, int S, int T, int d,
+             int V, float* __restrict__ dW) {
+  extern __shared__ float smem[];
+  float* w = smem;                     // [d]
+  __shared__ float dzc[kF32Threads];
+  const int v = blockIdx.x;
+  const int tid = threadIdx.x;
+  for (int k = tid; k < d; k += kF32Threads) w[k] = W[static_cast<size_t>(v) * d + k];
+  float acc[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+  const long long P = static_cast<long long>(S) * T;
+  for (long long p0 = 0; p0 < P; p0 += kF32Threads) {
+    __syncthreads();
+    const long long pos = p0 + tid;
+    float dzv = 0.f;
+    if (pos < P && mask[pos] != 0) {
+      const float* hr = H + pos * d;
+      float z = 0.f;
+      for (int k = 0; k < d; ++k) z = fmaf(w[k], hr[k], z);
+      const float pr = expf(z - lse[pos]);
+      dzv = g[pos] * ((tokens[pos] == v ? 1.f : 0.f) - pr);
+    }
+    dzc[tid] = dzv;
+    __syncthreads();
+    const long long rem = P - p0;
+    const int cnt = rem < kF32Threads ? static_cast<int>(rem) : kF32Threads;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int k = tid + j * kF32Threads;
+      if (k < d) {
+        float a = acc[j];
+        for (int q = 0; q < cnt; ++q) {
+          const float c = dzc[q];
+          if (c != 0.f) a = fmaf(c, H[(p0 + q) * d + k], a);
+        }
+        acc[j] = a;
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const int k = tid + j * kF32Threads;
+    if (k < d) dW[static_cast<size_t>(v) * d + k] = acc[j];
+  }
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------------------------
+// launches
+// ------------------------------------------------------------------------------------------
+cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
+                             int32_t* seq_last, cudaStream_t st) {
+  const int warps = 8;
+  k_mask_scan<<<(S + warps - 1) / warps, warps * 32, 0, st>>>(mask, S, T, counts, seq_last);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tile_list(const int32_t* seq_last, const int32_t* counts, int S, int T,
+                             int32_t* seq_tile_base, int2* tiles, WsHeader* hdr, cudaStream_t st) {
+  k_tile_list<<<1, 1024, 0, st>>>(seq_last, counts, S, T, seq_tile_base, tiles, hdr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_adv(const float* rewards, const int32_t* go, int num_groups, int S,
+                             int std_mode, float std_eps, float* adv, WsHeader* hdr,
+                             cudaStream_t st) {
+  k_group_adv<<<num_groups, 32, 0, st>>>(rewards, go, num_groups, S, std_mode, std_eps, adv, hdr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num_strips,
+                             const float* zy, const int32_t* seq_tile_base,
+                             const int32_t* tokens, const uint8_t* mask, int S, int T, int V,
+                             float* logp, float* lse, float* entropy, int32_t* argmax,
+                             WsHeader* hdr, cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  const int threads = 256;
+  k_fwd_merge<<<static_cast<unsigned>((P + threads - 1) / threads), threads, 0, st>>>(
+      partials, rows_cap, num_strips, zy, seq_tile_base, tokens, mask, S, T, V, logp, lse,
+      entropy, argmax, hdr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const float* old_logp,
+                               const float* ref_logp, const float* adv,
+                               const int32_t* valid_count, int S, int T, float eps_low,
+                               float eps_high, float beta, int agg, double norm,
+                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st) {
+  k_loss_tokens<<<S, kLossThreads, 0, st>>>(mask, logp, old_logp, ref_logp, adv, valid_count, S,
+                                            T, eps_low, eps_high, beta, agg, norm, hdr, g,
+                                            seq_loss);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm,
+                              const WsHeader* hdr, float* loss_out, cudaStream_t st) {
+  (void)agg;
+  (void)norm;
+  (void)hdr;
+  k_loss_final<<<1, 1024, 0, st>>>(seq_loss, S, loss_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d,
+                                __nv_bfloat16* dH, cudaStream_t st) {
+  dim3 grid((T + kTileRows - 1) / kTileRows, S);
+  k_dh_zero_tail<<<grid, 256, 0, st>>>(seq_tile_base, S, T, d, dH);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_f32_fwd(const float* H, const float* W, const int32_t* tokens,
+                           const uint8_t* mask, int S, int T, int d, int V, float* logp,
+                           float* lse, float* entropy, int32_t* argmax, WsHeader* hdr,
+                           cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  k_f32_fwd<<<static_cast<unsigned>(P), kF32Threads, d * sizeof(float), st>>>(
+      H, W, tokens, mask, S, T, d, V, logp, lse, entropy, argmax, hdr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_f32_dh(const float* H, const float* W, const int32_t* tokens,
+                          const uint8_t* mask, const float* lse, const float* g, int S, int T,
+                          int d, int V, float* dH, cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  const size_t sm = (static_cast<size_t>(d) + kF32VChunk) * sizeof(float);
+  k_f32_dh<<<static_cast<unsigned>(P), kF32Threads, sm, st>>>(H, W, tokens, mask, lse, g, S, T,
+                                                              d, V, dH);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
+                          const uint8_t* mask, const float* lse, const float* g, int S, int T,
+                          int d, int V, float* dW, cudaStream_t st) {
+  k_f32_dw<<<V, kF32Threads, d * sizeof(float), st>>>(H, W, tokens, mask, lse, g, S, T, d, V, dW);
+  return cudaGetLastError();
+}
+
+}  // namespace grpo

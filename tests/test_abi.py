@@ -1,0 +1,71 @@
+"""The C-ABI library builds for sm_103a, loads, exports every function include/grpo.h declares,
+and rejects bad arguments on the host before touching the GPU (no GPU needed)."""
+import ctypes
+
+import pytest
+
+import __graft_entry__
+from paper_2510_17158_gb300 import grpo as G
+
+
+@pytest.fixture(scope="module")
+def lib():
+    __graft_entry__.build()
+    return G._lib()
+
+
+def test_exports_every_declared_function(lib):
+    names = G.header_functions()
+    assert "grpo_score_fwd" in names and "grpo_loss_bwd" in names and "group_advantages" in names
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_kernel_names(lib):
+    for st in range(-7, 1):
+        assert G.grpo_status_string(st) != "unknown status"
+    assert [G.grpo_kernel_name(k) for k in range(len(G.KERNEL_NAMES))] == G.KERNEL_NAMES
+
+
+def test_workspace_bytes(lib):
+    S, T, d, V = 32, 16384, 5120, 151936
+    full = G.grpo_workspace_bytes(S, T, d, V, G.GRPO_BF16, 0)
+    rows = S * 128 * 128
+    assert full >= rows * 152064 * 2                 # whole-vocabulary dz scratch
+    small = G.grpo_workspace_bytes(S, T, d, V, G.GRPO_BF16, 8192)
+    assert small < full and small >= rows * 8192 * 2 + rows * d * 4
+    assert G.grpo_workspace_bytes(0, T, d, V, G.GRPO_BF16, 0) == 0
+    assert G.grpo_workspace_bytes(4, 64, 64, 512, G.GRPO_F32, 0) > 0
+
+
+def test_host_validation_rejects_before_launch(lib):
+    nul = ctypes.c_void_p(0)
+    st = lib.grpo_score_fwd(nul, nul, 1, nul, nul, 4, 64, 256, 512, nul, nul, nul, nul, nul, nul,
+                            1 << 20, nul)
+    assert st == -1
+    fake = ctypes.c_void_p(1 << 20)      # never dereferenced: validation fails first
+    # d not a multiple of 256 is unsupported on the bf16 tensor-core path
+    st = lib.grpo_score_fwd(fake, fake, 1, fake, fake, 4, 64, 320, 512, fake, fake, fake, fake,
+                            fake, fake, 1 << 30, nul)
+    assert st == -2
+    # misaligned workspace
+    st = lib.grpo_score_fwd(fake, fake, 1, fake, fake, 4, 64, 256, 512, fake, fake, fake, fake,
+                            fake, ctypes.c_void_p((1 << 20) + 8), 1 << 30, nul)
+    assert st == -4
+    # ref_logp NULL with beta > 0
+    st = lib.grpo_loss_bwd(fake, fake, 1, fake, fake, 4, 64, 256, 512, fake, fake, fake, nul,
+                           fake, fake, 0.2, 0.2, 0.04, 0, 0.0, fake, fake, fake, fake, 1 << 30, nul)
+    assert st == -1
+    # bad aggregation mode
+    st = lib.grpo_loss_bwd(fake, fake, 1, fake, fake, 4, 64, 256, 512, fake, fake, fake, fake,
+                           fake, fake, 0.2, 0.2, 0.04, 7, 0.0, fake, fake, fake, fake, 1 << 30, nul)
+    assert st == -1
+    # workspace too small
+    st = lib.grpo_loss_bwd(fake, fake, 1, fake, fake, 4, 64, 256, 512, fake, fake, fake, fake,
+                           fake, fake, 0.2, 0.2, 0.04, 0, 0.0, fake, fake, fake, fake, 1024, nul)
+    assert st == -4
+    # group advantages: bad std mode, no workspace
+    st = lib.group_advantages(fake, fake, 2, 8, 5, 1e-4, fake, fake, 1024, nul)
+    assert st == -1
+    st = lib.group_advantages(fake, fake, 2, 8, 0, 1e-4, fake, nul, 1024, nul)
+    assert st == -4

@@ -1,0 +1,114 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU float64 oracle on seeded inputs.
+
+Oracle-sized cases keep each workload's hidden size d, vocabulary V, dtype and value laws but
+fewer / shorter completions, so that they still span several 128-token tiles, many 256-column
+vocabulary tiles and the ragged tails (V % 256 = 128 for V = 151936; T % 128 != 0).
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2510_17158_gb300.synthetic import WORKLOADS, make_batch_numpy
+from tests.parity_util import compare, oracle_inputs, run_gpu, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+CASES = {
+    # name: (workload, overrides)
+    "tiny_f32": ("tiny_f32", {}),
+    "d2048_v32k": ("g8_t1k_d2048_v32k", dict(T=300, len_lo=64, len_hi=300)),
+    "d4096_v152k": ("g8_t4k_d4096_v152k", dict(group_sizes=(4,), T=160, len_lo=40, len_hi=160)),
+    "d5120_v152k_temp": ("g16_t16k_d5120_v152k",
+                         dict(group_sizes=(4,), prompts=1, T=144, len_lo=36, len_hi=144)),
+    "d3584_v152k_deg": ("g8_t512_d3584_v152k",
+                        dict(prompts=2, T=72, len_lo=16, len_hi=72, degenerate_frac=0.5)),
+}
+
+
+def _batch(name):
+    wname, over = CASES[name]
+    return make_batch_numpy(WORKLOADS[wname].scaled(**over))
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_parity_workload(name):
+    b = _batch(name)
+    w = b.workload
+    old, ref = oracle_inputs(b)
+    g = run_gpu(b, old, ref, w.eps, w.eps, w.beta)
+    o = run_oracle(b, old, ref, w.eps, w.eps, w.beta)
+    rep = compare(b, g, o)
+    print(name, rep)
+
+
+def test_parity_interior_holes_and_wide_ratio_noise():
+    """Tool-result spans masked inside completions; old-logp noise sigma 0.3 so that ~30% of
+    the tokens sit outside the clip range (both clip branches exercised)."""
+    w = WORKLOADS["g8_t1k_d2048_v32k"].scaled(T=200, len_lo=64, len_hi=200, holes=True)
+    b = make_batch_numpy(w)
+    old, ref = oracle_inputs(b, old_scale=6.0)
+    g = run_gpu(b, old, ref, 0.2, 0.28, 0.04)
+    o = run_oracle(b, old, ref, 0.2, 0.28, 0.04)
+    print(compare(b, g, o))
+
+
+def test_parity_token_mean_population_std():
+    b = _batch("d2048_v32k")
+    old, ref = oracle_inputs(b)
+    g = run_gpu(b, old, ref, 0.2, 0.2, 0.04, agg="token_mean", std_mode="population")
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04, agg="token_mean", std_mode="population")
+    print(compare(b, g, o))
+
+
+def test_parity_chunked_backward_matches_single_chunk():
+    """A workspace that holds only 4096 vocabulary columns of dz runs the backward in chunks with
+    an f32 dH accumulator; results match the oracle and the one-chunk run."""
+    b = _batch("d2048_v32k")
+    old, ref = oracle_inputs(b)
+    g1 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+    gc = run_gpu(b, old, ref, 0.2, 0.2, 0.04, vocab_chunk=4096)
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
+    print(compare(b, gc, o))
+    assert np.array_equal(g1["dW"].numpy(), gc["dW"].numpy())
+
+
+@pytest.mark.parametrize("eps,beta", [(0.1, 0.0), (0.1, 0.04), (0.2, 0.0), (0.2, 0.04),
+                                      (0.3, 0.0), (0.3, 0.04)])
+def test_parity_eps_beta_grid(eps, beta):
+    b = make_batch_numpy(WORKLOADS["g8_t512_d3584_v152k"].scaled(prompts=1, T=48, len_lo=16,
+                                                                   len_hi=48))
+    old, ref = oracle_inputs(b, old_scale=2.0)
+    g = run_gpu(b, old, ref, eps, eps, beta, ref_none=(beta == 0.0))
+    o = run_oracle(b, old, ref, eps, eps, beta)
+    print(compare(b, g, o))
+
+
+def test_group_advantages_mixed_group_sizes():
+    """64 prompts with G cycling {4, 8, 12, 16} and 10% degenerate groups (advantages only)."""
+    from paper_2510_17158_gb300 import grpo as G
+    import oracle
+    w = WORKLOADS["mixed_t512_d3584_v152k"]
+    rng = np.random.default_rng(7)
+    sizes = [w.group_sizes[p % 4] for p in range(w.prompts)]
+    go = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int32)
+    r = rng.uniform(-1, 3, size=go[-1]).astype(np.float32)
+    for g in rng.choice(len(sizes), size=6, replace=False):
+        r[go[g]:go[g + 1]] = r[go[g]]
+    ws = G.Workspace.create(256)
+    for mode in ("unbiased", "population"):
+        a = G.group_advantages(torch.from_numpy(r).cuda(), torch.from_numpy(go).cuda(), ws,
+                               std_mode=mode).cpu().numpy()
+        o = oracle.group_advantages(r, go, mode, 1e-4)
+        np.testing.assert_allclose(a, o, rtol=1e-5, atol=2e-6)
+        assert np.all(a[o == 0] == 0)
+    assert G.grpo_last_device_error(ws)[0] == 0
+
+
+def test_deterministic_bitwise():
+    b = _batch("d2048_v32k")
+    old, ref = oracle_inputs(b)
+    g1 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+    g2 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+    for k in ("logp", "lse", "entropy", "argmax", "dH", "dW"):
+        assert torch.equal(g1[k], g2[k]), k
+    assert g1["loss"] == g2["loss"]
