@@ -1,0 +1,396 @@
+"""Throughput of one fused GRPO update step (scoring + loss + backward) on GB300.
+
+A step is the whole path over one synthetic batch: group_advantages -> grpo_score_fwd ->
+grpo_loss_bwd (logits, log-softmax at the sampled token, entropy, argmax, advantages, clipped
+surrogate + KL loss, dL/dH and dL/dW). Default workload: 2 prompts x G=16 completions, T=16384,
+lengths U{4096..16384}, d=5120, V=151936, bf16, per-token temperature U[0.5, 2].
+
+Metric: scored tokens per second (fwd+bwd) and the algorithmic TFLOP/s (6 N d V per step) as a
+fraction of the measured dense BF16 peak. Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N --steps K --warmup W --config NAME]
+  python bench.py --impl reference ...   # the CPU float64 oracle on host cores, same metric
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+DEFAULT_CONFIG = "g16_t16k_d5120_v152k"
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+PROFILES = os.path.join(ROOT, "profiles")
+KERNEL_SRC = os.path.join(ROOT, "paper_2510_17158_gb300", "csrc", "gemm_tc.cu")
+GEMM_KERNELS = ("fwd_gemm_tc", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc")
+
+
+def peaks():
+    try:
+        p = json.load(open(PEAKS_PATH))
+        return {"hbm_gbs": p["hbm_gbs"], "bf16": p["bf16_tflops"],
+                "bf16_sustained": p["bf16_tflops_sustained"], "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def dist_init(ws, backend):
+    if ws > 1:
+        import torch.distributed as dist
+        if not dist.is_initialized():
+            dist.init_process_group(backend=backend)
+
+
+def dist_max(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def dist_sum(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples every 200 ms while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                rows.append((float(f[1]), float(f[2]), float(f[3]), f[5], f[6], f[7], f[8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        reasons = set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in loaded:
+            for n, v in zip(names, r[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in rows), "samples": len(loaded),
+                "power_w_max": max(r[2] for r in rows), "reasons": sorted(reasons)}
+
+
+def kernel_source_sha() -> str:
+    return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary of this kernel, if it was taken on the
+    current kernel source (profiles/<kernel>__<workload>.md with 'source_sha' and
+    'dram_bytes_per_launch_full' lines)."""
+    path = os.path.join(PROFILES, f"{kernel}__{workload}.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    sha = re.search(r"source_sha:\s*([0-9a-f]+)", txt)
+    val = re.search(r"dram_bytes_per_launch_full:\s*([0-9.eE+]+)", txt)
+    if not sha or not val or sha.group(1) != kernel_source_sha():
+        return None
+    return float(val.group(1))
+
+
+def apply_scale(w, spec: str):
+    if not spec:
+        return w
+    kw = {}
+    for item in spec.split(","):
+        k, v = item.split("=")
+        kw[k] = tuple(int(x) for x in v.split("/")) if k == "group_sizes" else int(v)
+    return w.scaled(name=w.name + "_scaled", **kw)
+
+
+# ---------------------------------------------------------------------------------------------
+def run_reference(args, ws_size, rank):
+    """The CPU float64 oracle, as it stands, timed on this host's cores on a bounded sample of the
+    workload (a slice of scored tokens of the first completion, full d and V)."""
+    if rank != 0:
+        return
+    from paper_2510_17158_gb300.synthetic import WORKLOADS
+    w = apply_scale(WORKLOADS[args.config], args.scale)
+    line = cpu_baseline(w, args.ref_tokens, steps=args.steps, warmup=args.warmup)
+    value = line["value"]
+    out = {"metric": "scored tokens/sec (fwd+bwd)", "value": value, "unit": "tokens/s",
+           "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": line["ms_per_step"], "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+           "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": w.T,
+                      "d": w.d, "V": w.V},
+           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": line["cores"],
+                            "kind": "oracle", "sample": line["sample"]},
+           "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def cpu_baseline(w, n_tokens, steps=1, warmup=0):
+    """Times oracle.grpo_step (fwd + loss + dH + full dW) on the first `n_tokens` positions of
+    one completion of workload `w` (inputs drawn with the workload's laws), float64 on host cores."""
+    import oracle
+    rng = np.random.default_rng(w.seed)
+    d, V = w.d, w.V
+    H = rng.standard_normal((1, n_tokens, d)).astype(np.float32)
+    H /= np.sqrt((H.astype(np.float64) ** 2).mean(-1, keepdims=True)).astype(np.float32)
+    if w.temperature:
+        H /= rng.uniform(*w.temperature, size=(1, n_tokens, 1)).astype(np.float32)
+    tdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    H = torch.from_numpy(H).to(tdt).double().numpy()
+    W = torch.from_numpy((rng.standard_normal((V, d), dtype=np.float32) * 0.02)).to(tdt).double().numpy()
+    tokens = rng.integers(0, V, size=(1, n_tokens)).astype(np.int32)
+    mask = np.ones((1, n_tokens), np.uint8)
+    old = rng.normal(-8, 1, size=(1, n_tokens))
+    ref = old + rng.normal(0, 0.1, size=(1, n_tokens))
+    rewards = np.array([1.0], np.float32)
+    go = np.array([0, 1], np.int32)
+    times = []
+    for it in range(warmup + steps):
+        t0 = time.perf_counter()
+        oracle.grpo_step(H, W, tokens, mask, rewards, go, old, ref, w.eps, w.eps, w.beta)
+        if it >= warmup:
+            times.append(time.perf_counter() - t0)
+    per = sum(times) / len(times)
+    return {"value": n_tokens / per, "ms_per_step": per * 1e3, "cores": os.cpu_count(),
+            "sample": f"{n_tokens} scored tokens of one completion, full d={d}, V={V} "
+                      f"(fwd + loss + dH + full dW), float64 numpy on {os.cpu_count()} host "
+                      f"threads; mean of {len(times)} run(s)"}
+
+
+# ---------------------------------------------------------------------------------------------
+def run_gpu(args):
+    ws_n, rank, local = dist_env()
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    dist_init(ws_n, "nccl")
+    from paper_2510_17158_gb300 import grpo as G
+    from paper_2510_17158_gb300.synthetic import WORKLOADS, lm_head_flops, make_batch_torch
+    w = apply_scale(WORKLOADS[args.config], args.scale)
+    w = w.scaled(seed=w.seed + 1000 * rank)        # each rank scores its own groups
+    t_gen = time.time()
+    b = make_batch_torch(w, device=str(device))
+    S, T, d, V = w.S, w.T, w.d, w.V
+    N_v = int(b.mask.sum().item())
+    ws = G.Workspace.for_problem(S, T, d, V, b.H.dtype, vocab_chunk=args.vocab_chunk,
+                                 device=device)
+    stream = torch.cuda.current_stream(device)
+    # old / ref log-probs: the policy's own log-prob (a scoring pass) plus the workload's noise
+    f0 = G.grpo_score_fwd(b.H, b.W, b.tokens, b.mask, ws)
+    old = (f0["logp"] + b.noise_old).contiguous()
+    ref = (f0["logp"] + b.noise_ref).contiguous()
+    fwd_out = {k: torch.empty_like(v) for k, v in f0.items()}
+    bwd_out = {"loss": torch.empty(1, device=device), "dH": torch.empty_like(b.H),
+               "dW": torch.empty((V, d), dtype=torch.float32, device=device)}
+    adv = torch.empty(S, device=device)
+    torch.cuda.synchronize()
+    gen_s = time.time() - t_gen
+
+    def step(H, W, tok, mask, rewards, go, old_, ref_):
+        G.group_advantages(rewards, go, ws, adv_out=adv)
+        f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
+        return G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_, ref_, adv,
+                               f["valid_count"], ws, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
+                               out=bwd_out)
+
+    dev_args = (b.H, b.W, b.tokens, b.mask, b.rewards, b.group_offsets, old, ref)
+    for _ in range(args.warmup):
+        step(*dev_args)
+    torch.cuda.synchronize()
+    st, where = G.grpo_last_device_error(ws)
+    if st != 0:
+        raise RuntimeError(f"device status {st} at {where} during warm-up")
+
+    # ---- device-resident timed region --------------------------------------------------------
+    G.grpo_timing_reset()
+    G.grpo_timing_enable(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(device.index if device.index is not None else 0) as clk:
+        barrier(ws_n)
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step(*dev_args)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier(ws_n)
+    G.grpo_timing_enable(False)
+    ms = ev0.elapsed_time(ev1)
+    ms_max = dist_max(ms, ws_n, device)
+    table = G.timing_table()
+    launches = sum(n for n, _ in table.values())
+    st, where = G.grpo_last_device_error(ws)
+    if st != 0:
+        raise RuntimeError(f"device status {st} at {where} in the timed region")
+
+    # ---- end to end through the public API with host buffers --------------------------------
+    host = {k: v.cpu().pin_memory() for k, v in zip(
+        ("H", "W", "tokens", "mask", "rewards", "go", "old", "ref"), dev_args)}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    e2e_steps = max(1, args.e2e_steps)
+    torch.cuda.synchronize()
+    barrier(ws_n)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        for k, dst in zip(host, dev_args):
+            dst.copy_(host[k], non_blocking=True)
+        r = step(*dev_args)
+        loss_host.copy_(r["loss"], non_blocking=True)
+        torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    barrier(ws_n)
+    e2e_s = dist_max(e2e_s, ws_n, device)
+
+    total_tokens = dist_sum(float(N_v), ws_n, device)
+    value = total_tokens * args.steps / (ms_max / 1e3)
+    e2e_value = total_tokens * e2e_steps / e2e_s
+    pk = peaks()
+    step_ms = ms_max / args.steps
+    alg_tflops = lm_head_flops(N_v, d, V) / (step_ms / 1e3) / 1e12
+
+    # ---- roofline of the dominant kernel -------------------------------------------------------
+    per_kernel = {k: {"launches": n, "ms_total": round(t, 3), "ms_per_launch": round(t / n, 4),
+                      "share": round(t / ms, 4)} for k, (n, t) in table.items()}
+    dom = max(table, key=lambda k: table[k][1])
+    n_dom, t_dom = table[dom]
+    chunk = args.vocab_chunk or V
+    flops_per_launch = {
+        "fwd_gemm_tc": 2.0 * N_v * d * V, "bwd_dz_gemm_tc": 2.0 * N_v * d * min(V, chunk),
+        "bwd_dh_gemm_tc": 2.0 * N_v * d * min(V, chunk), "bwd_dw_gemm_tc": 2.0 * N_v * d * min(V, chunk)}
+    if dom in flops_per_launch:
+        achieved = flops_per_launch[dom] / ((t_dom / n_dom) / 1e3) / 1e12
+        roof = {"kernel": dom, "bound": "tensor", "achieved": round(achieved, 1),
+                "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+                "frac": round(achieved / pk["bf16_sustained"], 4),
+                "peak_source": f"{pk['source']} bf16 sustained (kernel timed inside a long step)",
+                "traffic": ncu_traffic(dom, w.name)}
+    else:
+        roof = {"kernel": dom, "bound": "hbm", "achieved": None, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": None, "traffic": None}
+    gemm_tf = {}
+    for k in GEMM_KERNELS:
+        if k in table:
+            n, t = table[k]
+            gemm_tf[k] = round(flops_per_launch[k] / ((t / n) / 1e3) / 1e12, 1)
+
+    out = {
+        "metric": "scored tokens/sec (fwd+bwd)", "value": round(value, 1), "unit": "tokens/s",
+        "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
+                   "d": d, "V": V, "scored_tokens_per_rank": N_v,
+                   "vocab_chunk": args.vocab_chunk or "whole vocabulary",
+                   "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
+                       b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
+                   "parallelism": f"dp{ws_n} (independent groups per GPU)"},
+        "tflops_alg": round(alg_tflops, 1),
+        "frac_of_bf16_peak": round(alg_tflops / pk["bf16"], 4),
+        "frac_of_bf16_sustained": round(alg_tflops / pk["bf16_sustained"], 4),
+        "gemm_tflops_alg": gemm_tf,
+        "roofline": roof,
+        "kernels": per_kernel,
+        "gpu_launches": launches,
+        "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": 4, "steps": e2e_steps},
+        "clocks": clk.summary(),
+        "setup_s": round(gen_s, 1),
+    }
+    if rank == 0 and ws_n == 1 and not args.no_cpu_baseline:
+        cb = cpu_baseline(w, args.cpu_tokens)
+        out["cpu_baseline"] = {"value": round(cb["value"], 2), "unit": "tokens/s",
+                               "cores": cb["cores"], "kind": "oracle", "sample": cb["sample"]}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--vocab-chunk", type=int, default=0)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--cpu-tokens", type=int, default=32)
+    ap.add_argument("--ref-tokens", type=int, default=16)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--scale", default="",
+                    help="override workload fields, e.g. 'prompts=1,group_sizes=2,T=2048' "
+                         "(for profiling captures on a smaller case)")
+    args = ap.parse_args()
+    if args.impl == "ours":
+        args.warmup = max(3, args.warmup)      # timing rule: at least 3 warm-up steps
+    ws_n, rank, _ = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws_n, rank)
+        return
+    run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()
