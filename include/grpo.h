@@ -90,6 +90,31 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
                    float* lse, float* entropy, int32_t* argmax, int32_t* valid_count,
                    void* workspace, size_t workspace_bytes, grpo_stream_t stream);
 
+/* Bytes of the library-owned device scratch array used by grpo_score_fwd_static. */
+#define GRPO_STATIC_SCRATCH_BYTES (64u * 1024u * 1024u)
+
+/* grpo_score_fwd without a workspace, for callers that cannot allocate device memory -- e.g. a
+ * plugin whose host framework owns every device allocation and forbids extensions from making
+ * their own, or a latency-critical section where an allocation (which can synchronise the
+ * device) is not allowed. The paper has no counterpart; this is a deployment convenience.
+ * Arguments, outputs and results are those of grpo_score_fwd, except:
+ *  - the scratch is a GRPO_STATIC_SCRATCH_BYTES (64 MiB) __device__ array inside the library,
+ *    held on every GPU that loads the library until the process exits. A batch whose scratch
+ *    (about 16 * S*ceil(T/128)*128 * ceil(V/2048) + 4*S*T bytes for bf16) does not fit returns
+ *    GRPO_ERR_WORKSPACE before anything is enqueued;
+ *  - it allocates nothing and calls no allocating routine;
+ *  - the first call made with a given device current looks up the array's device address
+ *    (cudaGetSymbolAddress) and caches it: make that first call before any stream capture;
+ *  - all calls share the one array and each overwrites it: calls that overlap on the GPU
+ *    (different streams, or different host threads on one device) race and corrupt each
+ *    other's results;
+ *  - the device status word (e.g. GRPO_ERR_TOKEN_RANGE) is cleared at the start of each call and
+ *    copied at its end into *status_out (one device int32; may be NULL). */
+int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                          const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                          float* logp, float* lse, float* entropy, int32_t* argmax,
+                          int32_t* valid_count, int32_t* status_out, grpo_stream_t stream);
+
 /* GRPO loss and its gradient (Eq. 1 with the clipped-ratio surrogate of Sec. 6.1; Alg. 1's
  * gradient step), per scored token t of sequence i:
  *   rho = exp(logp - old_logp);  surr = min(rho A_i, clip(rho, 1-eps_low, 1+eps_high) A_i)

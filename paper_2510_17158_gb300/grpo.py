@@ -59,6 +59,8 @@ def _declare(lib):
         "grpo_timing_reset": (ctypes.c_int, []),
         "grpo_timing_read": (ctypes.c_int, [_i32, ctypes.POINTER(_i64), ctypes.POINTER(_f64)]),
         "grpo_debug_inject_stall": (ctypes.c_int, [_i32]),
+        "grpo_score_fwd_static": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
+                                                 _p, _p, _p, _p, _p, _p]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -234,6 +236,33 @@ def grpo_loss_bwd(H, W, tokens, mask, logp, lse, old_logp, ref_logp, adv, valid_
                               AGG_MODES[agg], float(norm), _ptr(out["loss"]), _ptr(out["dH"]),
                               _ptr(out["dW"]), ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "grpo_loss_bwd")
+    return out
+
+
+def grpo_score_fwd_static(H: torch.Tensor, W: torch.Tensor, tokens: torch.Tensor,
+                          mask: torch.Tensor, out: Optional[dict] = None, stream=None) -> dict:
+    """grpo_score_fwd with the library's fixed device scratch instead of a workspace (for callers
+    that cannot allocate device memory). Adds out["status"], a device int32 status word."""
+    S, T, d = H.shape
+    V = W.shape[0]
+    code = _dtype_code(H)
+    _need(H, "H", H.dtype)
+    _need(W, "W", H.dtype, (V, d))
+    _need(tokens, "tokens", torch.int32, (S, T))
+    _need(mask, "mask", torch.uint8, (S, T))
+    if out is None:
+        f = dict(dtype=torch.float32, device=H.device)
+        out = {"logp": torch.empty((S, T), **f), "lse": torch.empty((S, T), **f),
+               "entropy": torch.empty((S, T), **f),
+               "argmax": torch.empty((S, T), dtype=torch.int32, device=H.device),
+               "valid_count": torch.empty((S,), dtype=torch.int32, device=H.device),
+               "status": torch.empty((1,), dtype=torch.int32, device=H.device)}
+    st = _lib().grpo_score_fwd_static(_ptr(H), _ptr(W), code, _ptr(tokens), _ptr(mask), S, T, d,
+                                      V, _ptr(out["logp"]), _ptr(out["lse"]),
+                                      _ptr(out["entropy"]), _ptr(out["argmax"]),
+                                      _ptr(out["valid_count"]), _ptr(out.get("status")),
+                                      _stream(stream))
+    _check(st, "grpo_score_fwd_static")
     return out
 
 
