@@ -404,6 +404,8 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
     } else {  // ROLE_DW
       const int vrow = m * BM + r;
       const bool rv = vrow < a.vc_len;
+      // No scored token at all (K = 0): no MMA ran, the accumulator holds nothing -> dW = 0.
+      const bool empty_k = dm.num_kb == 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
       float* dst_row = a.dW + static_cast<size_t>(a.vc0 + vrow) * a.d + n * BN;
@@ -411,6 +413,10 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
         if (!rv) continue;
+        if (empty_k) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) x[j] = 0.f;
+        }
         float4* dst = reinterpret_cast<float4*>(dst_row + c * 32);
 #pragma unroll
         for (int j = 0; j < 8; ++j)

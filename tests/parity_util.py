@@ -35,16 +35,17 @@ def oracle_inputs(batch, old_scale=1.0):
 
 
 def run_oracle(batch, old, ref, eps_low, eps_high, beta, agg="seq_mean", std_mode="unbiased",
-               std_eps=1e-4, with_grads=True, vocab_rows=None):
+               std_eps=1e-4, with_grads=True, vocab_rows=None, norm=None):
     return oracle.grpo_step(batch.H.cpu().double().numpy(), batch.W.cpu().double().numpy(),
                             batch.tokens.cpu().numpy(), batch.mask.cpu().numpy(),
                             batch.rewards.cpu().numpy(), batch.group_offsets.cpu().numpy(),
                             old.astype(np.float64), ref.astype(np.float64), eps_low, eps_high, beta,
-                            agg, std_mode, std_eps, with_grads=with_grads, vocab_rows=vocab_rows)
+                            agg, std_mode, std_eps, norm=norm, with_grads=with_grads,
+                            vocab_rows=vocab_rows)
 
 
 def run_gpu(batch, old, ref, eps_low, eps_high, beta, agg="seq_mean", std_mode="unbiased",
-            std_eps=1e-4, vocab_chunk=0, ref_none=False, device="cuda"):
+            std_eps=1e-4, vocab_chunk=0, ref_none=False, device="cuda", norm=0.0):
     from paper_2510_17158_gb300 import grpo as G
     dev = torch.device(device)
     H, W = batch.H.to(dev), batch.W.to(dev)
@@ -59,7 +60,7 @@ def run_gpu(batch, old, ref, eps_low, eps_high, beta, agg="seq_mean", std_mode="
     ref_t = None if ref_none else torch.from_numpy(ref).to(dev)
     r = G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_t, ref_t, adv,
                         f["valid_count"], ws, eps_low=eps_low, eps_high=eps_high, beta=beta,
-                        agg=agg)
+                        agg=agg, norm=norm)
     torch.cuda.synchronize()
     st, where = G.grpo_last_device_error(ws)
     out = {k: v.cpu() for k, v in f.items()}
