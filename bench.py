@@ -228,6 +228,7 @@ def run_gpu(args):
     dist_init(ws_n, "nccl")
     from paper_2510_17158_gb300 import grpo as G
     from paper_2510_17158_gb300.synthetic import WORKLOADS, lm_head_flops, make_batch_torch
+    G.grpo_set_cta_pair(bool(args.cta_pair))
     w = apply_scale(WORKLOADS[args.config], args.scale)
     w = w.scaled(seed=w.seed + 1000 * rank)        # each rank scores its own groups
     t_gen = time.time()
@@ -344,6 +345,8 @@ def run_gpu(args):
         "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
                    "d": d, "V": V, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
+                   "tiles": "CTA pair 256x256 (cta_group::2)" if args.cta_pair else
+                            "single CTA 128x256 (cta_group::1)",
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
                        b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
                    "parallelism": f"dp{ws_n} (independent groups per GPU)"},
@@ -379,6 +382,8 @@ def main():
     ap.add_argument("--cpu-tokens", type=int, default=32)
     ap.add_argument("--ref-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cta-pair", type=int, default=0,
+                    help="tensor-core tiles: 0 = single CTAs (default), 1 = CTA pairs (cta_group::2)")
     ap.add_argument("--scale", default="",
                     help="override workload fields, e.g. 'prompts=1,group_sizes=2,T=2048' "
                          "(for profiling captures on a smaller case)")

@@ -163,6 +163,13 @@ int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms);
  * such a call are undefined. Process-wide; not for production use. */
 int grpo_debug_inject_stall(int32_t on);
 
+/* Tensor-core tile shape of the four LM-head GEMMs, process-wide, for launches made afterwards:
+ * on == 0 (default): one CTA per 128 x 256 tile (tcgen05 cta_group::1); on != 0: CTA pairs --
+ * clusters of two CTAs on one TPC compute 256 x 256 tiles with cta_group::2, each CTA staging
+ * half of B. Results agree within rounding. The pair mode does more work per clock, but on a
+ * power-capped GB300 it draws more power per flop, so the single-CTA mode is the default. */
+int grpo_set_cta_pair(int32_t on);
+
 #ifdef __cplusplus
 }
 #endif

@@ -30,6 +30,7 @@ struct EventPair {
 std::mutex g_mu;
 std::atomic<int> g_timing{0};
 std::atomic<int> g_inject_stall{0};
+std::atomic<int> g_cta_pair{0};   // tensor-core tiles: 1 = CTA pairs (cta_group::2), 0 = single CTAs
 std::atomic<long long> g_launches[GRPO_K_COUNT];
 std::vector<EventPair> g_pending[GRPO_K_COUNT];
 double g_total_ms[GRPO_K_COUNT];
@@ -171,10 +172,18 @@ int num_sms() {
   return n;
 }
 
-int gemm_grid(long long units) {
+// Persistent grid for `row_units` x `col_units` output tiles of 128 rows: one CTA per SM, or
+// one CTA pair per two SMs (then rows are paired and the grid is even).
+int gemm_grid(long long row_units, long long col_units, bool pair) {
   const long long sms = num_sms();
-  if (sms <= 0) return 1;
-  return static_cast<int>(units < sms ? (units > 0 ? units : 1) : sms);
+  if (sms <= 1) return pair ? 2 : 1;
+  if (!pair) {
+    const long long u = row_units * col_units;
+    return static_cast<int>(u < sms ? (u > 0 ? u : 1) : sms);
+  }
+  const long long pairs = ((row_units + 1) / 2) * col_units;
+  const long long cap = sms / 2;
+  return static_cast<int>(2 * (pairs < cap ? (pairs > 0 ? pairs : 1) : cap));
 }
 
 struct Views {
@@ -314,16 +323,17 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
     return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
   }));
+  const bool pair = g_cta_pair.load() != 0;
   CUtensorMap mapH, mapW;
   if (!make_map(&mapH, H, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
-      !make_map(&mapW, W, d, V, d, kTileN))
+      !make_map(&mapW, W, d, V, d, pair ? kTileN / 2 : kTileN))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
   a.partials = v.partials;
   a.zy = v.zy;
-  const int grid = gemm_grid(static_cast<long long>(L.max_tiles) * L.num_strips);
+  const int grid = gemm_grid(L.max_tiles, L.num_strips, pair);
   GRPO_TRY(counted(GRPO_K_FWD_GEMM, st,
-                   [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, st); }));
+                   [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st); }));
   return counted(GRPO_K_FWD_MERGE, st, [&] {
     return launch_fwd_merge(v.partials, L.rows_cap, L.num_strips, v.zy, v.seq_tile_base, tokens,
                             mask, S, T, V, logp, lse, entropy, argmax, v.hdr, st);
@@ -405,9 +415,11 @@ int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* to
     dz = reinterpret_cast<__nv_bfloat16*>(wsb + L.fixed_end +
                                           align256(static_cast<size_t>(L.rows_cap) * d * 4));
   }
+  const bool pair = g_cta_pair.load() != 0;
   CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn;
   const uint64_t P = static_cast<uint64_t>(S) * T;
-  if (!make_map(&mapHk, H, d, P, d, kTileRows) || !make_map(&mapWk, W, d, V, d, kTileN) ||
+  if (!make_map(&mapHk, H, d, P, d, kTileRows) ||
+      !make_map(&mapWk, W, d, V, d, pair ? kTileN / 2 : kTileN) ||
       !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
       !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
       !make_map(&mapHmn, H, d, P, d, 64))
@@ -427,15 +439,15 @@ int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* to
     a.dh_mode = nchunks == 1 ? 0 : (c == 0 ? 1 : (c == nchunks - 1 ? 3 : 2));
     const long long vt = (a.vc_len + kTileN - 1) / kTileN;
     GRPO_TRY(counted(GRPO_K_BWD_DZ_GEMM, st, [&] {
-      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles * vt), st);
+      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, pair), pair, st);
     }));
     GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
-      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a,
-                         gemm_grid(static_cast<long long>(L.max_tiles) * (d / kTileN)), st);
+      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, d / kTileN, pair),
+                         pair, st);
     }));
     const long long vm = (a.vc_len + kTileRows - 1) / kTileRows;
     GRPO_TRY(counted(GRPO_K_BWD_DW_GEMM, st, [&] {
-      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm * (d / kTileN)), st);
+      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, d / kTileN, pair), pair, st);
     }));
   }
   return counted(GRPO_K_DH_ZERO_TAIL, st, [&] {
@@ -495,5 +507,18 @@ int grpo_debug_inject_stall(int32_t on) {
   g_inject_stall.store(on ? 1 : 0);
   return GRPO_OK;
 }
+
+int grpo_set_cta_pair(int32_t on) {
+  g_cta_pair.store(on ? 1 : 0);
+  return GRPO_OK;
+}
+
+}  // extern "C"
+
+namespace grpo {
+bool gemm_pair_mode() { return g_cta_pair.load() != 0; }
+}  // namespace grpo
+
+extern "C" {
 
 }  // extern "C"

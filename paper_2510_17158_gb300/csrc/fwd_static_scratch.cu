@@ -148,9 +148,10 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
   } else {
     rc = ok_or_cuda(launch_tile_list(seq_last, valid_count, S, T, seq_tile_base, tiles, hdr, st));
     if (rc != GRPO_OK) return rc;
+    const bool pair = gemm_pair_mode();
     CUtensorMap mapH, mapW;
     if (!bf16_map(&mapH, H, d, static_cast<uint64_t>(S) * T, kTileRows) ||
-        !bf16_map(&mapW, W, d, V, kTileN))
+        !bf16_map(&mapW, W, d, V, pair ? kTileN / 2 : kTileN))
       return GRPO_ERR_CUDA;
     GemmArgs a;
     std::memset(&a, 0, sizeof(a));
@@ -170,9 +171,16 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return GRPO_ERR_CUDA;
-    const long long units = static_cast<long long>(L.max_tiles) * L.num_strips;
-    const int grid = static_cast<int>(units < sms ? (units > 0 ? units : 1) : sms);
-    rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, st));
+    int grid;
+    if (pair) {
+      const long long pairs = ((L.max_tiles + 1) / 2) * static_cast<long long>(L.num_strips);
+      const long long cap = sms / 2 > 0 ? sms / 2 : 1;
+      grid = static_cast<int>(2 * (pairs < cap ? (pairs > 0 ? pairs : 1) : cap));
+    } else {
+      const long long units = static_cast<long long>(L.max_tiles) * L.num_strips;
+      grid = static_cast<int>(units < sms ? (units > 0 ? units : 1) : sms);
+    }
+    rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st));
     if (rc != GRPO_OK) return rc;
     rc = ok_or_cuda(launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, seq_tile_base,
                                      tokens, mask, S, T, V, logp, lse, entropy, argmax, hdr, st));

@@ -9,11 +9,12 @@
 //   role DH  : dH = dz W (K = vocabulary chunk), f32 accumulation, written in H's dtype.
 //   role DW  : dW = dz^T H (K = tokens), f32.
 //
-// Block = 6 warps: warp 0 issues TMA loads into a 4-stage shared-memory ring, warp 1 issues
-// tcgen05.mma (M=128, N=256, K=16, bf16 in, f32 accumulate in tensor memory), warps 2-5 read
-// the accumulator back with tcgen05.ld (one TMEM lane = one output row per thread) and run the
-// role's epilogue. Two 256-column accumulators in TMEM let the epilogue of one tile overlap the
-// MMAs of the next. Every wait is bounded (see mbar_wait_bounded).
+// Block = 6 warps: warp 0 issues TMA loads into a shared-memory ring, warp 1 issues tcgen05.mma
+// (bf16 in, f32 accumulate in tensor memory), warps 2-5 read the accumulator back with
+// tcgen05.ld (one TMEM lane = one output row per thread) and run the role's epilogue. Two
+// 256-column accumulators in TMEM let the epilogue of one tile overlap the MMAs of the next.
+// Two modes: one CTA per 128 x 256 tile (cta_group::1), or a CTA pair per 256 x 256 tile
+// (cta_group::2, see Cfg). Every wait is bounded (see mbar_wait_bounded).
 #include <cfloat>
 
 #include "common.cuh"
@@ -22,18 +23,32 @@
 namespace grpo {
 namespace {
 
-constexpr int BM = kTileRows;  // 128
+constexpr int BM = kTileRows;  // 128 accumulator rows per CTA
 constexpr int BN = kTileN;     // 256
 constexpr int BK = 64;         // one 128-byte swizzle row of bf16
-constexpr int STAGES = 4;
-constexpr uint32_t A_STAGE = BM * BK * 2;  // 16 KB
-constexpr uint32_t B_STAGE = BN * BK * 2;  // 32 KB
-constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;
 constexpr uint32_t BOX_MN = 64 * 64 * 2;   // one 64 x 64 bf16 box (MN-major operands)
 constexpr uint32_t TMEM_COLS = 512;        // two 128 x 256 f32 accumulators
 constexpr int NUM_THREADS = 192;
-constexpr int GROUP_M = 16;                // raster: 16 row tiles share each column sweep
-constexpr size_t SMEM_BYTES = size_t(STAGES) * STAGE_TX + 1024 + 256;
+#ifndef GRPO_GROUP_M
+#define GRPO_GROUP_M 16
+#endif
+constexpr int GROUP_M = GRPO_GROUP_M;      // raster: row units sharing each column sweep
+
+// PAIR = false: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128).
+// PAIR = true : a CTA pair (cluster of 2 on one TPC) computes a 256 x 256 tile with
+//               cta_group::2 (M = 256): each CTA stages its 128 rows of A and half (128 rows)
+//               of B, so per-SM operand traffic for B halves and the ring can be 6 deep.
+template <bool PAIR>
+struct Cfg {
+  static constexpr int STAGES = PAIR ? 6 : 4;
+  static constexpr uint32_t A_STAGE = BM * BK * 2;                      // 16 KB
+  static constexpr uint32_t B_ROWS = PAIR ? BN / 2 : BN;                // B rows staged here
+  static constexpr uint32_t B_STAGE = B_ROWS * BK * 2;                  // 16 or 32 KB
+  static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;               // bytes per CTA
+  static constexpr size_t SMEM = size_t(STAGES) * STAGE_TX + 1024 + 256;
+};
+constexpr size_t SMEM_BYTES = Cfg<false>::SMEM > Cfg<true>::SMEM ? Cfg<false>::SMEM
+                                                                  : Cfg<true>::SMEM;
 
 struct Dims {
   int num_m, num_n, num_kb;
@@ -83,25 +98,54 @@ __device__ __forceinline__ int acc_tiles_of_unit(const GemmArgs& a, int n) {
   return 1;
 }
 
+// Work layout shared by the three roles of a CTA. In PAIR mode a unit is a pair of M tiles
+// (2*mu for the leader CTA, 2*mu + 1 for its peer) and the pairs are strided over clusters.
+template <bool PAIR>
+struct Sched {
+  int rank;        // CTA rank in the pair (0 = leader, issues the MMAs); 0 without PAIR
+  int first, step; // unit loop: u = first; u < num_units; u += step
+  int num_mu, num_units;
+
+  __device__ __forceinline__ Sched(const Dims& dm) {
+    rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;
+    first = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+    step = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
+    num_mu = PAIR ? (dm.num_m + 1) / 2 : dm.num_m;
+    num_units = num_mu * dm.num_n;
+  }
+  // M tile of this CTA for unit row mu; `ok` false for the missing half of an odd tail pair
+  // (then `load` names a valid tile to stage, and nothing is stored).
+  __device__ __forceinline__ void m_of(int mu, int num_m, int& m, int& load, bool& ok) const {
+    m = PAIR ? 2 * mu + rank : mu;
+    ok = m < num_m;
+    load = ok ? m : (PAIR ? 2 * mu : mu);
+  }
+};
+
 // ------------------------------------------------------------------------------------------
-// producer: one thread
+// producer: one thread per CTA
 // ------------------------------------------------------------------------------------------
-template <int ROLE>
+template <int ROLE, bool PAIR>
 __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB, const GemmArgs& a,
-                             const Dims& dm, uint8_t* sA, uint8_t* sB, uint64_t* full,
-                             uint64_t* empty, volatile int* abort_flag) {
-  const int num_units = dm.num_m * dm.num_n;
-  const bool stall = (a.inject_stall != 0) && blockIdx.x == 0;
+                             const Dims& dm, const Sched<PAIR>& sc, uint8_t* sA, uint8_t* sB,
+                             uint64_t* full, uint64_t* empty, volatile int* abort_flag) {
+  using C = Cfg<PAIR>;
+  const bool leader = sc.rank == 0;
+  const bool stall = (a.inject_stall != 0) && blockIdx.x == 0;   // CTA 0 is a leader
+  constexpr int B_BOXES = static_cast<int>(C::B_ROWS) / 64;      // MN-major B boxes per stage
+  const int b_col0 = PAIR ? sc.rank * static_cast<int>(C::B_ROWS) : 0;
   uint32_t stage = 0, phase = 0;
   long long issued = 0;
   bool ok = true;
-  for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x) {
-    int m, n;
-    decode_unit(u, dm.num_m, dm.num_n, m, n);
+  for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
+    int mu, n, m, m_load;
+    bool m_ok;
+    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
+    sc.m_of(mu, dm.num_m, m, m_load, m_ok);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     int hrow = 0;
     if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
-      const int2 tl = a.tiles[m];
+      const int2 tl = a.tiles[m_load];
       hrow = tl.x * a.T + tl.y;
     }
     for (int t = 0; t < nacc && ok; ++t) {
@@ -111,69 +155,83 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB, c
           ok = false;
           break;
         }
-        const uint32_t dA = smem_u32(sA + stage * A_STAGE);
-        const uint32_t dB = smem_u32(sB + stage * B_STAGE);
+        const uint32_t dA = smem_u32(sA + stage * C::A_STAGE);
+        const uint32_t dB = smem_u32(sB + stage * C::B_STAGE);
+        // completion of both CTAs' copies is counted on the leader's barrier
+        const uint32_t bar = PAIR ? mapa_shared(smem_u32(&full[stage]), 0)
+                                  : smem_u32(&full[stage]);
+        auto load = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
+          if (PAIR) {
+            tma_load_2d_pair(dst, map, bar, x, y);
+          } else {
+            tma_load_2d(dst, map, &full[stage], x, y);
+          }
+        };
         if (stall && issued == 0) {
           // test hook: leave stage 0 unfilled so that the MMA warp's bounded wait runs out
         } else {
-          mbar_arrive_expect_tx(&full[stage], STAGE_TX);
+          if (leader) mbar_arrive_expect_tx(&full[stage], PAIR ? 2 * C::STAGE_TX : C::STAGE_TX);
           if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
             const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
-            tma_load_2d(dA, mapA, &full[stage], kb * BK, hrow);
-            tma_load_2d(dB, mapB, &full[stage], kb * BK, vt * BN);
+            load(dA, mapA, kb * BK, hrow);
+            load(dB, mapB, kb * BK, vt * BN + b_col0);
           } else if (ROLE == ROLE_DH) {
-            tma_load_2d(dA, mapA, &full[stage], kb * BK, m * BM);
+            load(dA, mapA, kb * BK, m_load * BM);
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j)
-              tma_load_2d(dB + j * BOX_MN, mapB, &full[stage], n * BN + j * 64, a.vc0 + kb * BK);
+            for (int j = 0; j < B_BOXES; ++j)
+              load(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kb * BK);
           } else {  // ROLE_DW
 #pragma unroll
             for (int j = 0; j < BM / 64; ++j)
-              tma_load_2d(dA + j * BOX_MN, mapA, &full[stage], m * BM + j * 64, kb * BK);
+              load(dA + j * BOX_MN, mapA, m_load * BM + j * 64, kb * BK);
             const int2 tl = a.tiles[kb >> 1];
             const int row = tl.x * a.T + tl.y + (kb & 1) * BK;
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j)
-              tma_load_2d(dB + j * BOX_MN, mapB, &full[stage], n * BN + j * 64, row);
+            for (int j = 0; j < B_BOXES; ++j)
+              load(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, row);
           }
         }
         ++issued;
-        if (++stage == STAGES) {
+        if (++stage == C::STAGES) {
           stage = 0;
           phase ^= 1u;
         }
       }
     }
   }
-  if (!ok) {
-    // Aborted: let the copies already in flight land before the CTA exits (bounded).
-    const long long back = issued < STAGES ? issued : STAGES;
+  if (!ok && leader) {
+    // Aborted: let the copies already in flight land before the CTA exits (bounded). In PAIR
+    // mode the leader's barriers also count the peer's copies; the peer waits for the leader
+    // at the final cluster barrier.
+    const long long back = issued < C::STAGES ? issued : C::STAGES;
     for (long long i = 1; i <= back; ++i) {
       const long long it = issued - i;
       if (stall && it == 0) continue;
-      const uint32_t s = static_cast<uint32_t>(it % STAGES);
-      const uint32_t ph = static_cast<uint32_t>((it / STAGES) & 1);
+      const uint32_t s = static_cast<uint32_t>(it % C::STAGES);
+      const uint32_t ph = static_cast<uint32_t>((it / C::STAGES) & 1);
       mbar_wait_drain(&full[s], ph, 100000000ull);
     }
   }
 }
 
 // ------------------------------------------------------------------------------------------
-// MMA issuer: one thread
+// MMA issuer: one thread (of the leader CTA in PAIR mode)
 // ------------------------------------------------------------------------------------------
-template <int ROLE>
-__device__ void run_mma(const GemmArgs& a, const Dims& dm, uint8_t* sA, uint8_t* sB,
-                        uint64_t* full, uint64_t* empty, uint64_t* accf, uint64_t* acce,
-                        uint64_t* drain, uint32_t tmem_base, volatile int* abort_flag) {
+template <int ROLE, bool PAIR>
+__device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc, uint8_t* sA,
+                        uint8_t* sB, uint64_t* full, uint64_t* empty, uint64_t* accf,
+                        uint64_t* acce, uint64_t* drain, uint32_t tmem_base,
+                        volatile int* abort_flag) {
+  using C = Cfg<PAIR>;
+  if (PAIR && sc.rank != 0) return;
   constexpr bool A_MN = (ROLE == ROLE_DW);
   constexpr bool B_MN = (ROLE == ROLE_DH || ROLE == ROLE_DW);
-  constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, A_MN, B_MN);
-  const int num_units = dm.num_m * dm.num_n;
+  constexpr uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * BM : BM, BN, A_MN, B_MN);
   uint32_t stage = 0, phase = 0, buf = 0, bphase = 0;
   bool ok = true;
-  for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x) {
-    int m, n;
-    decode_unit(u, dm.num_m, dm.num_n, m, n);
+  for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
+    int mu, n;
+    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     for (int t = 0; t < nacc && ok; ++t) {
       if (!mbar_wait_bounded(&acce[buf], bphase ^ 1u, abort_flag, a.hdr,
@@ -190,46 +248,77 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, uint8_t* sA, uint8_t*
           break;
         }
         tc_fence_after();
-        const uint32_t a0 = smem_u32(sA + stage * A_STAGE);
-        const uint32_t b0 = smem_u32(sB + stage * B_STAGE);
+        const uint32_t a0 = smem_u32(sA + stage * C::A_STAGE);
+        const uint32_t b0 = smem_u32(sB + stage * C::B_STAGE);
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k) {
           const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, BOX_MN, 1024)
                                    : sdesc_sw128(a0 + k * 32, 16, 1024);
           const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, BOX_MN, 1024)
                                    : sdesc_sw128(b0 + k * 32, 16, 1024);
-          umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          if (PAIR) {
+            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          } else {
+            umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          }
         }
-        umma_commit(&empty[stage]);  // frees the smem stage once these MMAs have read it
-        if (++stage == STAGES) {
+        // frees the smem stage (in both CTAs of a pair) once these MMAs have read it
+        if (PAIR) {
+          umma_commit_pair(&empty[stage], 0x3);
+        } else {
+          umma_commit(&empty[stage]);
+        }
+        if (++stage == C::STAGES) {
           stage = 0;
           phase ^= 1u;
         }
       }
       if (!ok) break;
-      umma_commit(&accf[buf]);       // accumulator ready for the epilogue
+      if (PAIR) {                      // accumulator ready for both CTAs' epilogues
+        umma_commit_pair(&accf[buf], 0x3);
+      } else {
+        umma_commit(&accf[buf]);
+      }
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
     }
   }
   // Make sure no MMA is still writing tensor memory when it is released.
-  umma_commit(drain);
+  if (PAIR) {
+    umma_commit_pair(drain, 0x1);
+  } else {
+    umma_commit(drain);
+  }
   mbar_wait_drain(drain, 0, 200000000ull);
 }
 
 // ------------------------------------------------------------------------------------------
 // epilogues: warps 2..5, thread = one accumulator row (TMEM lane)
 // ------------------------------------------------------------------------------------------
+#ifndef GRPO_EPI_SLEEP_NS
+#define GRPO_EPI_SLEEP_NS 20000
+#endif
+// Epilogue warps wait for a whole tile's MMAs (tens of microseconds to milliseconds): they sleep
+// in hardware between checks rather than keep four schedulers busy polling.
 __device__ __forceinline__ bool epi_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                          WsHeader* hdr, int32_t where) {
-  const bool ok = mbar_wait_bounded(bar, parity, abort_flag, hdr, where);
+  const bool ok = mbar_wait_bounded(bar, parity, abort_flag, hdr, where, GRPO_EPI_SLEEP_NS);
   return __all_sync(0xffffffffu, ok);
 }
 
-__device__ __forceinline__ void epi_release(uint64_t* bar, int lane) {
+// Tells the MMA issuer that this warp has read accumulator `bar`'s buffer; in PAIR mode the
+// barrier lives in the leader CTA and counts the epilogue warps of both CTAs.
+template <bool PAIR>
+__device__ __forceinline__ void epi_release(uint64_t* bar, int lane, int rank) {
   tc_fence_before();
   __syncwarp();
-  if (lane == 0) mbar_arrive(bar);
+  if (lane == 0) {
+    if (PAIR && rank != 0) {
+      mbar_arrive_cluster(mapa_shared(smem_u32(bar), 0));
+    } else {
+      mbar_arrive(bar);
+    }
+  }
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -237,23 +326,25 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
-template <int ROLE>
-__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, uint64_t* acce,
-                             uint32_t tmem_base, volatile int* abort_flag) {
+template <int ROLE, bool PAIR>
+__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc,
+                             uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
+                             volatile int* abort_flag) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;               // TMEM lane quadrant this warp may access
   const int r = q * 32 + lane;          // accumulator row of this thread
   const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-  const int num_units = dm.num_m * dm.num_n;
   const int32_t where = WHERE_GEMM_BASE + ROLE * 16 + 4;
   uint32_t buf = 0, bphase = 0;
-  for (int u = blockIdx.x; u < num_units; u += gridDim.x) {
-    int m, n;
-    decode_unit(u, dm.num_m, dm.num_n, m, n);
+  for (int u = sc.first; u < sc.num_units; u += sc.step) {
+    int mu, n, m, m_load;
+    bool m_ok;
+    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
+    sc.m_of(mu, dm.num_m, m, m_load, m_ok);
 
     if (ROLE == ROLE_FWD) {
-      const int2 tl = a.tiles[m];
-      const bool rv = tl.y + r < a.T;
+      const int2 tl = a.tiles[m_load];
+      const bool rv = m_ok && tl.y + r < a.T;
       const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
       const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] : -1;
       float rm = -INFINITY, rs = 0.f, ru = 0.f, zyv = 0.f;
@@ -285,9 +376,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
             }
           }
           if (cm > rm) {  // strictly greater: earlier (lower) index wins ties
-            const float sc = ex2_approx((rm - cm) * kLog2e);
-            rs *= sc;
-            ru *= sc;
+            const float scl = ex2_approx((rm - cm) * kLog2e);
+            rs *= scl;
+            ru *= scl;
             rm = cm;
             ri = v0 + ci;
           }
@@ -311,17 +402,18 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
             found = true;
           }
         }
-        epi_release(&acce[buf], lane);
+        epi_release<PAIR>(&acce[buf], lane, sc.rank);
         buf ^= 1u;
         if (buf == 0) bphase ^= 1u;
       }
-      a.partials[static_cast<long long>(n) * a.rows_cap + static_cast<long long>(m) * BM + r] =
-          make_float4(rm, rs, ru, __int_as_float(ri));
+      if (m_ok)
+        a.partials[static_cast<long long>(n) * a.rows_cap + static_cast<long long>(m) * BM + r] =
+            make_float4(rm, rs, ru, __int_as_float(ri));
       if (found) a.zy[pos] = zyv;
 
     } else if (ROLE == ROLE_DZ) {
-      const int2 tl = a.tiles[m];
-      const bool rv = tl.y + r < a.T;
+      const int2 tl = a.tiles[m_load];
+      const bool rv = m_ok && tl.y + r < a.T;
       const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
       const bool act = rv && a.mask[pos] != 0;
       const float gt = act ? a.g[pos] : 0.f;
@@ -330,12 +422,13 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
       __nv_bfloat16* dst_row =
-          a.dz + (static_cast<size_t>(m) * BM + r) * static_cast<size_t>(a.dz_pitch);
+          a.dz + (static_cast<size_t>(m_load) * BM + r) * static_cast<size_t>(a.dz_pitch);
       for (int c = 0; c < BN / 32; ++c) {
         const int vloc = n * BN + c * 32;
         const int v0 = a.vc0 + vloc;
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
+        if (!m_ok) continue;
         uint32_t pk[16];
         if (act) {
 #pragma unroll
@@ -356,13 +449,13 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
         for (int j = 0; j < 4; ++j)
           dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
       }
-      epi_release(&acce[buf], lane);
+      epi_release<PAIR>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
 
     } else if (ROLE == ROLE_DH) {
-      const int2 tl = a.tiles[m];
-      const bool rv = tl.y + r < a.T;
+      const int2 tl = a.tiles[m_load];
+      const bool rv = m_ok && tl.y + r < a.T;
       const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
@@ -397,13 +490,13 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
                                 pack_bf16x2(x[8 * j + 6], x[8 * j + 7]));
         }
       }
-      epi_release(&acce[buf], lane);
+      epi_release<PAIR>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
 
     } else {  // ROLE_DW
       const int vrow = m * BM + r;
-      const bool rv = vrow < a.vc_len;
+      const bool rv = m_ok && vrow < a.vc_len;
       // No scored token at all (K = 0): no MMA ran, the accumulator holds nothing -> dW = 0.
       const bool empty_k = dm.num_kb == 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
@@ -422,7 +515,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
         for (int j = 0; j < 8; ++j)
           dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
       }
-      epi_release(&acce[buf], lane);
+      epi_release<PAIR>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
     }
@@ -430,21 +523,21 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, uint64_t* accf, 
 }
 
 // ------------------------------------------------------------------------------------------
-// kernel
+// kernel body (both modes) and the two kernels
 // ------------------------------------------------------------------------------------------
-template <int ROLE>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
-    tc_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-            const __grid_constant__ GemmArgs args) {
+template <int ROLE, bool PAIR>
+__device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtensorMap* mapB,
+                                          const GemmArgs& args) {
+  using C = Cfg<PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * A_STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + STAGES * B_STAGE);
+  uint8_t* sB = smem + C::STAGES * C::A_STAGE;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_STAGE);
   uint64_t* full = bars;
-  uint64_t* empty = bars + STAGES;
-  uint64_t* accf = bars + 2 * STAGES;
+  uint64_t* empty = bars + C::STAGES;
+  uint64_t* accf = bars + 2 * C::STAGES;
   uint64_t* acce = accf + 2;
   uint64_t* drain = acce + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -452,13 +545,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], 4);
+      mbar_init(&acce[b], PAIR ? 8 : 4);  // epilogue warps of one or both CTAs
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -466,41 +559,87 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_proxy_async_smem();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapB);
+    tma_prefetch_desc(mapA);
+    tma_prefetch_desc(mapB);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(tmem_slot, TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR) {
+    cluster_sync_all();  // barriers of both CTAs initialised before any cross-CTA traffic
+  } else {
+    __syncthreads();
+  }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const Dims dm = role_dims<ROLE>(args, args.hdr->num_tiles);
+  const Sched<PAIR> sc(dm);
 
   if (warp == 0) {
-    if (lane == 0) run_producer<ROLE>(&mapA, &mapB, args, dm, sA, sB, full, empty, abort_flag);
+    if (lane == 0)
+      run_producer<ROLE, PAIR>(mapA, mapB, args, dm, sc, sA, sB, full, empty, abort_flag);
   } else if (warp == 1) {
     if (lane == 0)
-      run_mma<ROLE>(args, dm, sA, sB, full, empty, accf, acce, drain, tmem_base, abort_flag);
+      run_mma<ROLE, PAIR>(args, dm, sc, sA, sB, full, empty, accf, acce, drain, tmem_base,
+                          abort_flag);
   } else {
-    run_epilogue<ROLE>(args, dm, accf, acce, tmem_base, abort_flag);
+    run_epilogue<ROLE, PAIR>(args, dm, sc, accf, acce, tmem_base, abort_flag);
   }
   __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  if (PAIR) {
+    cluster_sync_all();  // no CTA leaves while its peer may still signal its barriers
+  } else {
+    __syncthreads();
+  }
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, TMEM_COLS);
+  if (warp == 1) {
+    if (PAIR) {
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    } else {
+      tmem_dealloc(tmem_base, TMEM_COLS);
+    }
+  }
+}
+
+template <int ROLE>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+            const __grid_constant__ GemmArgs args) {
+  gemm_body<ROLE, false>(&mapA, &mapB, args);
+}
+
+template <int ROLE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_pair(const __grid_constant__ CUtensorMap mapA,
+                 const __grid_constant__ CUtensorMap mapB, const __grid_constant__ GemmArgs args) {
+  gemm_body<ROLE, true>(&mapA, &mapB, args);
 }
 
 template <int ROLE>
 cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const GemmArgs& args,
-                        int grid, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(tc_gemm<ROLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(SMEM_BYTES));
-  if (e != cudaSuccess) return e;
-  tc_gemm<ROLE><<<grid, NUM_THREADS, SMEM_BYTES, st>>>(mapA, mapB, args);
+                        int grid, bool pair, cudaStream_t st) {
+  if (pair) {
+    const size_t smem = Cfg<true>::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair<ROLE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    tc_gemm_pair<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+  } else {
+    const size_t smem = Cfg<false>::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm<ROLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    tc_gemm<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+  }
   return cudaGetLastError();
 }
 
@@ -509,12 +648,12 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
 size_t gemm_smem_bytes() { return SMEM_BYTES; }
 
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, cudaStream_t st) {
+                        const GemmArgs& args, int grid, bool pair, cudaStream_t st) {
   switch (role) {
-    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, st);
-    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, st);
-    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, st);
-    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, st);
+    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, pair, st);
+    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, pair, st);
+    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, pair, st);
+    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, pair, st);
     default: return cudaErrorInvalidValue;
   }
 }

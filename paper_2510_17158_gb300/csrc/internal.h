@@ -84,9 +84,13 @@ cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
                           const uint8_t* mask, const float* lse, const float* g, int S, int T,
                           int d, int V, float* dW, cudaStream_t st);
 
+// Process-wide tensor-core tile mode chosen through grpo_set_cta_pair (true = CTA pairs).
+bool gemm_pair_mode();
+
 // tcgen05 GEMM launches. `grid` = persistent CTAs.
 size_t gemm_smem_bytes();
+// pair = true: CTA-pair kernels (clusters of 2, cta_group::2); `grid` must then be even.
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, cudaStream_t st);
+                        const GemmArgs& args, int grid, bool pair, cudaStream_t st);
 
 }  // namespace grpo

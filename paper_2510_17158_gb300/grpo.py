@@ -59,6 +59,7 @@ def _declare(lib):
         "grpo_timing_reset": (ctypes.c_int, []),
         "grpo_timing_read": (ctypes.c_int, [_i32, ctypes.POINTER(_i64), ctypes.POINTER(_f64)]),
         "grpo_debug_inject_stall": (ctypes.c_int, [_i32]),
+        "grpo_set_cta_pair": (ctypes.c_int, [_i32]),
         "grpo_score_fwd_static": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                                  _p, _p, _p, _p, _p, _p]),
     }
@@ -297,6 +298,10 @@ def grpo_timing_read(kid: int):
 
 def grpo_debug_inject_stall(on: bool):
     _check(_lib().grpo_debug_inject_stall(1 if on else 0), "grpo_debug_inject_stall")
+
+
+def grpo_set_cta_pair(on: bool):
+    _check(_lib().grpo_set_cta_pair(1 if on else 0), "grpo_set_cta_pair")
 
 
 def timing_table() -> dict:

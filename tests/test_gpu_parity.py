@@ -112,3 +112,21 @@ def test_deterministic_bitwise():
     for k in ("logp", "lse", "entropy", "argmax", "dH", "dW"):
         assert torch.equal(g1[k], g2[k]), k
     assert g1["loss"] == g2["loss"]
+
+
+def test_pair_tiles_match_oracle_and_single_cta_tiles():
+    """The CTA-pair tile mode (M = 256, cta_group::2) and the default 1-CTA mode (M = 128,
+    cta_group::1) both meet the parity bar and agree with each other."""
+    from paper_2510_17158_gb300 import grpo as G
+    b = _batch("d4096_v152k")
+    old, ref = oracle_inputs(b)
+    G.grpo_set_cta_pair(True)
+    try:
+        g1 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+    finally:
+        G.grpo_set_cta_pair(False)
+    g2 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
+    print(compare(b, g1, o), compare(b, g2, o))
+    for k in ("logp", "lse", "entropy"):
+        assert float((g1[k] - g2[k]).abs().max()) <= 1e-4
