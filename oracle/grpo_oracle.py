@@ -28,7 +28,9 @@ Readings of points the paper leaves open (each one is a documented choice):
   ``sum l / sum n``; masked tokens (padding, tool-result text) are not scored;
 * the subgradient of the clipped surrogate takes the unclipped branch when it is active with
   inclusive boundaries: active iff (A >= 0 and rho <= 1+eps_hi) or (A < 0 and rho >= 1-eps_lo);
-* argmax ties go to the lowest vocabulary index; entropy is in nats.
+* argmax ties go to the lowest vocabulary index; entropy is in nats;
+* distillation (Sec. 6.2) is token cross-entropy with the same aggregation choices;
+* the performance reward's "correct but slower" is t > t_base.
 
 Every input is converted exactly to float64 (bf16 and fp32 values are exactly representable).
 """
@@ -150,6 +152,40 @@ def aggregate(ell, dell, seq_of_token, counts, num_seqs, agg=SEQ_MEAN, norm=None
     return L, g, mass
 
 
+def sft_objective(logp):
+    """Sec. 6.2 (reasoning distillation): the small model is fine-tuned with supervised learning
+    on the large model's filtered traces, tool-call tokens and arguments kept in the targets, i.e.
+    token cross-entropy l_t = -log pi(y_t) over the target tokens. Returns l_t and dl/dlogp = -1."""
+    logp = _f64(logp)
+    return {"ell": -logp, "dell": -np.ones_like(logp)}
+
+
+def perf_reward(correct, t_base, t_new):
+    """Eq. 3: -2 if the edit is incorrect, -1 if correct but slower than the baseline, else
+    min{10, t_base / t - 1}. "Slower" is read as t > t_base (an unchanged time earns 0)."""
+    correct = np.asarray(correct) != 0
+    t_base, t_new = _f64(t_base), _f64(t_new)
+    out = np.empty(np.broadcast(correct, t_base, t_new).shape)
+    for i in np.ndindex(out.shape):
+        if not correct[i]:
+            out[i] = -2.0
+        elif t_new[i] > t_base[i]:
+            out[i] = -1.0
+        else:
+            out[i] = min(10.0, t_base[i] / t_new[i] - 1.0)
+    return out
+
+
+def tool_reward(tools_used, tools_avail, lam=0.5):
+    """Eq. 4: lambda_tools * |UniqueToolsUsed(x)| / |T_avail| with lambda_tools = 0.5."""
+    return lam * _f64(tools_used) / _f64(tools_avail)
+
+
+def reward(correct, t_base, t_new, tools_used, tools_avail, lam=0.5):
+    """Eq. 2: r(x) = r_perf(x) + r_tools(x)."""
+    return perf_reward(correct, t_base, t_new) + tool_reward(tools_used, tools_avail, lam)
+
+
 def logit_grads(h, W, y, lse, g):
     """dL/dz_t = g_t (onehot(y_t) - softmax(z_t)) for each scored token (chain rule through
     logp_t = z_t[y_t] - lse_t)."""
@@ -173,6 +209,33 @@ def param_grads(h, W, y, lse, g, vocab_rows=None):
     else:
         dW = dZ[:, vocab_rows].T @ _f64(h)
     return dH, dW
+
+
+def sft_step(H, W, tokens, mask, agg=TOKEN_MEAN, norm=None, vocab_rows=None, with_grads=True):
+    """The distillation (SFT) path of Sec. 6.2 on a padded batch: per-position logp etc. as in
+    grpo_step, L = mean token cross-entropy, dH [S,T,d] and dW [V,d]."""
+    H = _f64(H)
+    S, T, d = H.shape
+    mask = np.asarray(mask)
+    counts = valid_counts(mask)
+    idx = np.argwhere(mask != 0)
+    si, ti = idx[:, 0], idx[:, 1]
+    h = H[si, ti]
+    y = np.asarray(tokens)[si, ti]
+    sc = score_tokens(h, W, y)
+    ob = sft_objective(sc["logp"])
+    L, g_tok, mass = aggregate(ob["ell"], ob["dell"], si, counts, S, agg, norm)
+    out = {"counts": counts, "loss": L, "loss_abs_mass": mass}
+    lp = np.zeros((S, T))
+    lp[si, ti] = sc["logp"]
+    out["logp"] = lp
+    if with_grads:
+        dHv, dW = param_grads(h, W, y, sc["lse"], g_tok, vocab_rows)
+        dH = np.zeros((S, T, d))
+        dH[si, ti] = dHv
+        out["dH"] = dH
+        out["dW"] = dW
+    return out
 
 
 def grpo_step(H, W, tokens, mask, rewards, group_offsets, old, ref, eps_low=0.2, eps_high=0.2,

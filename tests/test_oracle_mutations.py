@@ -31,6 +31,13 @@ MUTATIONS = [
     ("argmax last index", "argmax = Z.argmax(axis=1) ", "argmax = Z.shape[1] - 1 - Z[:, ::-1].argmax(axis=1) "),
     ("ratio inverted", "rho = np.exp(logp - old)", "rho = np.exp(old - logp)"),
     ("counts of zeros", "return (m != 0).sum(axis=1)", "return (m == 0).sum(axis=1)"),
+    ("sft gradient sign", "return {\"ell\": -logp, \"dell\": -np.ones_like(logp)}",
+     "return {\"ell\": -logp, \"dell\": np.ones_like(logp)}"),
+    ("reward cap", "out[i] = min(10.0, t_base[i] / t_new[i] - 1.0)",
+     "out[i] = min(10.0, t_base[i] / t_new[i])"),
+    ("slower penalty", "out[i] = -1.0", "out[i] = -2.0"),
+    ("tool reward ratio inverted", "return lam * _f64(tools_used) / _f64(tools_avail)",
+     "return lam * _f64(tools_avail) / _f64(tools_used)"),
 ]
 
 

@@ -301,10 +301,42 @@ def pin_counts(o):
     assert list(o.valid_counts(mask)) == brute
 
 
+def pin_sft_torch_cross_entropy(o):
+    """Sec. 6.2 distillation loss = torch's cross_entropy (mean over target tokens), and its
+    gradients through the LM head equal torch float64 autograd; uniform logits give log V."""
+    b = make_batch_numpy(WORKLOADS["tiny_f32"])
+    H, W = b.H.double().numpy(), b.W.double().numpy()
+    mask = b.mask.numpy()
+    tok = b.tokens.numpy()
+    out = o.sft_step(H, W, tok, mask)
+    idx = np.argwhere(mask != 0)
+    th = torch.tensor(H[idx[:, 0], idx[:, 1]], requires_grad=True)
+    tW = torch.tensor(W, requires_grad=True)
+    L = torch.nn.functional.cross_entropy(th @ tW.T, torch.tensor(tok[idx[:, 0], idx[:, 1]]).long())
+    L.backward()
+    assert abs(L.item() - out["loss"]) < 1e-12
+    np.testing.assert_allclose(out["dH"][idx[:, 0], idx[:, 1]], th.grad.numpy(), rtol=1e-9,
+                               atol=1e-15)
+    np.testing.assert_allclose(out["dW"], tW.grad.numpy(), rtol=1e-9, atol=1e-15)
+    u = o.sft_step(H, np.zeros_like(W), tok, mask, with_grads=False)
+    assert abs(u["loss"] - math.log(W.shape[0])) < 1e-12
+
+
+def pin_golden_rewards(o):
+    for c in json.load(open(GOLDEN))["rewards"]:
+        rp = o.perf_reward(np.array([c["correct"]]), np.array([c["t_base"]]), np.array([c["t_new"]]))
+        rt = o.tool_reward(np.array([c["tools_used"]]), np.array([c["tools_avail"]]))
+        r = o.reward(np.array([c["correct"]]), np.array([c["t_base"]]), np.array([c["t_new"]]),
+                     np.array([c["tools_used"]]), np.array([c["tools_avail"]]))
+        assert abs(rp[0] - c["r_perf"]) < 1e-12 and abs(rt[0] - c["r_tools"]) < 1e-12, c["why"]
+        assert abs(r[0] - c["r"]) < 1e-12, c["why"]
+
+
 PINS = [pin_uniform_logits, pin_scipy_log_softmax, pin_scipy_entropy, pin_argmax_ties,
         pin_golden_objective, pin_golden_advantages, pin_advantages_scipy_and_invariants,
         pin_finite_differences, pin_on_policy_reinforce, pin_torch_autograd,
-        pin_dW_rows_sum_to_zero, pin_vocab_row_subset, pin_counts]
+        pin_dW_rows_sum_to_zero, pin_vocab_row_subset, pin_counts, pin_sft_torch_cross_entropy,
+        pin_golden_rewards]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
