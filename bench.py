@@ -250,6 +250,10 @@ def run_gpu(args):
     gen_s = time.time() - t_gen
 
     def step(H, W, tok, mask, rewards, go, old_, ref_):
+        if args.path == "sft":       # distillation step (Sec. 6.2): no advantages, no ratio
+            f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
+            return G.grpo_sft_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], f["valid_count"],
+                                       ws, out=bwd_out)
         G.group_advantages(rewards, go, ws, adv_out=adv)
         f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
         return G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_, ref_, adv,
@@ -338,8 +342,9 @@ def run_gpu(args):
             gemm_tf[k] = round(flops_per_launch[k] / ((t / n) / 1e3) / 1e12, 1)
 
     out = {
-        "metric": "scored tokens/sec (fwd+bwd)", "value": round(value, 1), "unit": "tokens/s",
-        "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
+        "metric": "scored tokens/sec (fwd+bwd)" + (" [SFT distillation step]" if args.path == "sft"
+                                                    else ""),
+        "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(step_ms, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
@@ -382,6 +387,8 @@ def main():
     ap.add_argument("--cpu-tokens", type=int, default=32)
     ap.add_argument("--ref-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--path", default="grpo", choices=["grpo", "sft"],
+                    help="grpo: the GRPO update (default); sft: the distillation loss step")
     ap.add_argument("--cta-pair", type=int, default=0,
                     help="tensor-core tiles: 0 = single CTAs (default), 1 = CTA pairs (cta_group::2)")
     ap.add_argument("--scale", default="",

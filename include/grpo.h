@@ -134,6 +134,29 @@ int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* to
                   float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
                   grpo_stream_t stream);
 
+/* Distillation loss and gradient (Sec. 6.2: the small model is fine-tuned by supervised
+ * learning on the large model's filtered traces, tool-call tokens kept in the targets): token
+ * cross-entropy l_t = -logp_t over the scored tokens, aggregated like grpo_loss_bwd
+ * (GRPO_AGG_TOKEN_MEAN is the usual choice), so g_t = -w_t; then the same recompute + dz + dH +
+ * dW contractions as grpo_loss_bwd. Arguments as in grpo_loss_bwd. */
+int grpo_sft_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                      const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                      const float* logp, const float* lse, const int32_t* valid_count,
+                      int32_t agg, double norm, float* loss_out, void* dH, float* dW,
+                      void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
+/* Rewards of n completions (Eq. 2: r = r_perf + r_tools), the input of group_advantages:
+ *   r_perf (Eq. 3) = -2 if correct[i] == 0; -1 if t_new[i] > t_base[i] (correct but slower);
+ *                    else min(10, t_base[i] / t_new[i] - 1)
+ *   r_tools (Eq. 4) = lambda_tools * tools_used[i] / tools_avail[i] (the paper: 0.5; unique
+ *                    tools used out of the 4-6 made available); NaN unless
+ *                    0 <= tools_used <= tools_avail and tools_avail >= 1.
+ * correct uint8 [n], t_base / t_new f32 [n] (seconds), tools_used / tools_avail int32 [n],
+ * r_out f32 [n]. */
+int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new,
+                 const int32_t* tools_used, const int32_t* tools_avail, int32_t n,
+                 float lambda_tools, float* r_out, grpo_stream_t stream);
+
 /* Synchronises `stream`, returns the first device-side status recorded in the workspace since
  * the last call (GRPO_OK if none) and clears it. *where_out (may be NULL) gets a code naming the
  * kernel and wait that recorded it. */
@@ -148,7 +171,7 @@ enum {
   GRPO_K_MASK_SCAN = 0, GRPO_K_TILE_LIST, GRPO_K_GROUP_ADV, GRPO_K_FWD_GEMM, GRPO_K_FWD_MERGE,
   GRPO_K_LOSS_TOKENS, GRPO_K_LOSS_FINAL, GRPO_K_BWD_DZ_GEMM, GRPO_K_BWD_DH_GEMM,
   GRPO_K_BWD_DW_GEMM, GRPO_K_DH_ZERO_TAIL, GRPO_K_F32_FWD, GRPO_K_F32_DH, GRPO_K_F32_DW,
-  GRPO_K_COUNT
+  GRPO_K_REWARDS, GRPO_K_COUNT
 };
 const char* grpo_kernel_name(int32_t kernel_id);
 int grpo_timing_enable(int32_t enable);   /* 1 = record events from now on, 0 = stop */

@@ -21,7 +21,7 @@ namespace {
 const char* const kKernelNames[GRPO_K_COUNT] = {
     "mask_scan",       "tile_list",    "group_adv",   "fwd_gemm_tc",  "fwd_merge",
     "loss_tokens",     "loss_final",   "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw"};
+    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw",      "rewards"};
 
 struct EventPair {
   cudaEvent_t a, b;
@@ -340,17 +340,29 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   });
 }
 
-int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+}  // extern "C"
+
+namespace {
+
+// Shared by grpo_loss_bwd (mode 0) and grpo_sft_loss_bwd (mode 1): the per-token loss kernel
+// differs, the recompute + dz + dH + dW GEMMs are the same.
+int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const int32_t* tokens,
                   const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
                   const float* logp, const float* lse, const float* old_logp,
                   const float* ref_logp, const float* adv, const int32_t* valid_count,
                   float eps_low, float eps_high, float beta, int32_t agg, double norm,
                   float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
                   grpo_stream_t stream) {
-  if (!H || !W || !tokens || !mask || !logp || !lse || !old_logp || !adv || !valid_count ||
-      !loss_out || !dH || !dW)
+  if (!H || !W || !tokens || !mask || !logp || !lse || !valid_count || !loss_out || !dH || !dW)
     return GRPO_ERR_INVALID_ARG;
-  if (!ref_logp && beta != 0.f) return GRPO_ERR_INVALID_ARG;
+  if (mode == 0 && (!old_logp || !adv)) return GRPO_ERR_INVALID_ARG;
+  if (mode == 0 && !ref_logp && beta != 0.f) return GRPO_ERR_INVALID_ARG;
+  if (mode != 0) {   // the distillation loss reads none of these
+    old_logp = logp;
+    ref_logp = logp;
+    adv = logp;
+    beta = 0.f;
+  }
   if (!shape_ok(S, T, d, V)) return GRPO_ERR_INVALID_ARG;
   GRPO_TRY(check_dtype_shape(dtype, d));
   if (agg != GRPO_AGG_SEQ_MEAN && agg != GRPO_AGG_TOKEN_MEAN) return GRPO_ERR_INVALID_ARG;
@@ -371,7 +383,7 @@ int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* to
   }));
   GRPO_TRY(counted(GRPO_K_LOSS_TOKENS, st, [&] {
     return launch_loss_tokens(mask, logp, old_logp, ref, adv, valid_count, S, T, eps_low,
-                              eps_high, beta, agg, norm, v.hdr, v.g, v.seq_loss, st);
+                              eps_high, beta, agg, norm, mode, v.hdr, v.g, v.seq_loss, st);
   }));
   GRPO_TRY(counted(GRPO_K_LOSS_FINAL, st, [&] {
     return launch_loss_final(v.seq_loss, S, agg, norm, v.hdr, loss_out, st);
@@ -452,6 +464,45 @@ int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* to
   }
   return counted(GRPO_K_DH_ZERO_TAIL, st, [&] {
     return launch_dh_zero_tail(v.seq_tile_base, S, T, d, static_cast<__nv_bfloat16*>(dH), st);
+  });
+}
+
+}  // namespace
+
+extern "C" {
+
+int grpo_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                  const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                  const float* logp, const float* lse, const float* old_logp,
+                  const float* ref_logp, const float* adv, const int32_t* valid_count,
+                  float eps_low, float eps_high, float beta, int32_t agg, double norm,
+                  float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
+                  grpo_stream_t stream) {
+  return loss_bwd_impl(0, H, W, dtype, tokens, mask, S, T, d, V, logp, lse, old_logp, ref_logp,
+                       adv, valid_count, eps_low, eps_high, beta, agg, norm, loss_out, dH, dW,
+                       workspace, workspace_bytes, stream);
+}
+
+int grpo_sft_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,
+                      const uint8_t* mask, int32_t S, int32_t T, int32_t d, int32_t V,
+                      const float* logp, const float* lse, const int32_t* valid_count,
+                      int32_t agg, double norm, float* loss_out, void* dH, float* dW,
+                      void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  return loss_bwd_impl(1, H, W, dtype, tokens, mask, S, T, d, V, logp, lse, nullptr, nullptr,
+                       nullptr, valid_count, 0.f, 0.f, 0.f, agg, norm, loss_out, dH, dW, workspace,
+                       workspace_bytes, stream);
+}
+
+int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new,
+                 const int32_t* tools_used, const int32_t* tools_avail, int32_t n,
+                 float lambda_tools, float* r_out, grpo_stream_t stream) {
+  if (!correct || !t_base || !t_new || !tools_used || !tools_avail || !r_out || n <= 0)
+    return GRPO_ERR_INVALID_ARG;
+  if (!(lambda_tools >= 0.f)) return GRPO_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  return counted(GRPO_K_REWARDS, st, [&] {
+    return launch_rewards(correct, t_base, t_new, tools_used, tools_avail, n, lambda_tools,
+                          r_out, st);
   });
 }
 

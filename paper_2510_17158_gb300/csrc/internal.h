@@ -67,8 +67,11 @@ cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num
 cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const float* old_logp,
                                const float* ref_logp, const float* adv,
                                const int32_t* valid_count, int S, int T, float eps_low,
-                               float eps_high, float beta, int agg, double norm,
+                               float eps_high, float beta, int agg, double norm, int mode,
                                const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st);
+cudaError_t launch_rewards(const uint8_t* correct, const float* t_base, const float* t_new,
+                           const int32_t* used, const int32_t* avail, int n, float lambda_tools,
+                           float* r, cudaStream_t st);
 cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm,
                               const WsHeader* hdr, float* loss_out, cudaStream_t st);
 cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d,

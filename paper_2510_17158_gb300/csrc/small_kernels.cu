@@ -233,15 +233,18 @@ __device__ __forceinline__ float block_sum_fixed(float v, float* sh) {
   return tot;  // valid in thread 0
 }
 
+// mode 0: GRPO clipped surrogate + KL (Sec. 6.1, Eq. 1); mode 1: distillation token
+// cross-entropy l_t = -logp_t (Sec. 6.2).
 __global__ void __launch_bounds__(kLossThreads)
     k_loss_tokens(const uint8_t* __restrict__ mask, const float* __restrict__ logp,
                   const float* __restrict__ old_logp, const float* __restrict__ ref_logp,
                   const float* __restrict__ adv, const int32_t* __restrict__ valid_count, int S,
                   int T, float eps_low, float eps_high, float beta, int agg, double norm,
-                  const WsHeader* hdr, float* __restrict__ g, float* __restrict__ seq_loss) {
+                  int mode, const WsHeader* hdr, float* __restrict__ g,
+                  float* __restrict__ seq_loss) {
   __shared__ float sh[32];
   const int i = blockIdx.x;
-  const float A = adv[i];
+  const float A = mode == 0 ? adv[i] : 0.f;
   const int n_i = valid_count[i];
   float w;
   if (agg == 0) {
@@ -257,7 +260,10 @@ __global__ void __launch_bounds__(kLossThreads)
   for (int t = threadIdx.x; t < T; t += kLossThreads) {
     const size_t pos = base + t;
     float gt = 0.f;
-    if (mask[pos] != 0) {
+    if (mask[pos] != 0 && mode == 1) {
+      acc -= logp[pos];
+      gt = -w;
+    } else if (mask[pos] != 0) {
       const float lp = logp[pos];
       const float rho = expf(lp - old_logp[pos]);
       const float unclipped = rho * A;
@@ -280,6 +286,29 @@ __global__ void __launch_bounds__(kLossThreads)
   }
   const float tot = block_sum_fixed(acc, sh);
   if (threadIdx.x == 0) seq_loss[i] = tot * w;
+}
+
+// Eqs. 2-4: r = r_perf + r_tools, r_perf = -2 (incorrect), -1 (correct, t > t_base),
+// else min(10, t_base / t - 1); r_tools = lambda * used / avail (NaN if the counts are invalid).
+__global__ void k_rewards(const uint8_t* __restrict__ correct, const float* __restrict__ t_base,
+                          const float* __restrict__ t_new, const int32_t* __restrict__ used,
+                          const int32_t* __restrict__ avail, int n, float lambda_tools,
+                          float* __restrict__ r) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float rp;
+  if (correct[i] == 0) {
+    rp = -2.f;
+  } else if (t_new[i] > t_base[i]) {
+    rp = -1.f;
+  } else {
+    rp = fminf(10.f, t_base[i] / t_new[i] - 1.f);
+  }
+  const int u = used[i], a = avail[i];
+  const float rt = (a > 0 && u >= 0 && u <= a)
+                       ? lambda_tools * static_cast<float>(u) / static_cast<float>(a)
+                       : __int_as_float(0x7fc00000);
+  r[i] = rp + rt;
 }
 
 __global__ void k_loss_final(const float* __restrict__ seq_loss, int S, float* loss_out) {
@@ -536,11 +565,19 @@ cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num
 cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const float* old_logp,
                                const float* ref_logp, const float* adv,
                                const int32_t* valid_count, int S, int T, float eps_low,
-                               float eps_high, float beta, int agg, double norm,
+                               float eps_high, float beta, int agg, double norm, int mode,
                                const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st) {
   k_loss_tokens<<<S, kLossThreads, 0, st>>>(mask, logp, old_logp, ref_logp, adv, valid_count, S,
-                                            T, eps_low, eps_high, beta, agg, norm, hdr, g,
+                                            T, eps_low, eps_high, beta, agg, norm, mode, hdr, g,
                                             seq_loss);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rewards(const uint8_t* correct, const float* t_base, const float* t_new,
+                           const int32_t* used, const int32_t* avail, int n, float lambda_tools,
+                           float* r, cudaStream_t st) {
+  k_rewards<<<(n + 255) / 256, 256, 0, st>>>(correct, t_base, t_new, used, avail, n,
+                                             lambda_tools, r);
   return cudaGetLastError();
 }
 

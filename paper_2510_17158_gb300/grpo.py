@@ -27,7 +27,7 @@ STATUS_NAMES = {0: "GRPO_OK", -1: "GRPO_ERR_INVALID_ARG", -2: "GRPO_ERR_UNSUPPOR
                 -6: "GRPO_ERR_TIMEOUT", -7: "GRPO_ERR_GROUPS"}
 KERNEL_NAMES = ["mask_scan", "tile_list", "group_adv", "fwd_gemm_tc", "fwd_merge", "loss_tokens",
                 "loss_final", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-                "dh_zero_tail", "f32_fwd", "f32_dh", "f32_dw"]
+                "dh_zero_tail", "f32_fwd", "f32_dh", "f32_dw", "rewards"]
 
 
 class GrpoError(RuntimeError):
@@ -60,6 +60,9 @@ def _declare(lib):
         "grpo_timing_read": (ctypes.c_int, [_i32, ctypes.POINTER(_i64), ctypes.POINTER(_f64)]),
         "grpo_debug_inject_stall": (ctypes.c_int, [_i32]),
         "grpo_set_cta_pair": (ctypes.c_int, [_i32]),
+        "grpo_sft_loss_bwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
+                                             _p, _p, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
+        "grpo_rewards": (ctypes.c_int, [_p, _p, _p, _p, _p, _i32, _f32, _p, _p]),
         "grpo_score_fwd_static": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                                  _p, _p, _p, _p, _p, _p]),
     }
@@ -265,6 +268,49 @@ def grpo_score_fwd_static(H: torch.Tensor, W: torch.Tensor, tokens: torch.Tensor
                                       _stream(stream))
     _check(st, "grpo_score_fwd_static")
     return out
+
+
+def grpo_sft_loss_bwd(H, W, tokens, mask, logp, lse, valid_count, ws: Workspace,
+                      agg="token_mean", norm=0.0, out: Optional[dict] = None, stream=None) -> dict:
+    """Distillation (token cross-entropy) loss and gradients; dict(loss, dH, dW)."""
+    S, T, d = H.shape
+    V = W.shape[0]
+    code = _dtype_code(H)
+    _need(H, "H", H.dtype)
+    _need(W, "W", H.dtype, (V, d))
+    _need(tokens, "tokens", torch.int32, (S, T))
+    _need(mask, "mask", torch.uint8, (S, T))
+    _need(logp, "logp", torch.float32, (S, T))
+    _need(lse, "lse", torch.float32, (S, T))
+    _need(valid_count, "valid_count", torch.int32, (S,))
+    if out is None:
+        out = {"loss": torch.empty((1,), dtype=torch.float32, device=H.device),
+               "dH": torch.empty_like(H),
+               "dW": torch.empty((V, d), dtype=torch.float32, device=H.device)}
+    st = _lib().grpo_sft_loss_bwd(_ptr(H), _ptr(W), code, _ptr(tokens), _ptr(mask), S, T, d, V,
+                                  _ptr(logp), _ptr(lse), _ptr(valid_count), AGG_MODES[agg],
+                                  float(norm), _ptr(out["loss"]), _ptr(out["dH"]),
+                                  _ptr(out["dW"]), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "grpo_sft_loss_bwd")
+    return out
+
+
+def grpo_rewards(correct, t_base, t_new, tools_used, tools_avail, lambda_tools=0.5,
+                 r_out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Eq. 2-4 rewards of n completions (device tensors)."""
+    n = correct.numel()
+    _need(correct, "correct", torch.uint8, (n,))
+    _need(t_base, "t_base", torch.float32, (n,))
+    _need(t_new, "t_new", torch.float32, (n,))
+    _need(tools_used, "tools_used", torch.int32, (n,))
+    _need(tools_avail, "tools_avail", torch.int32, (n,))
+    if r_out is None:
+        r_out = torch.empty((n,), dtype=torch.float32, device=correct.device)
+    st = _lib().grpo_rewards(_ptr(correct), _ptr(t_base), _ptr(t_new), _ptr(tools_used),
+                             _ptr(tools_avail), n, float(lambda_tools), _ptr(r_out),
+                             _stream(stream))
+    _check(st, "grpo_rewards")
+    return r_out
 
 
 def grpo_last_device_error(ws: Workspace, stream=None):
