@@ -107,6 +107,40 @@ def score_tokens(h, W, y):
             "second": second}
 
 
+def shard_stats(h, W_shard, y, v_offset):
+    """Vocabulary-parallel scoring (the paper shards the policy with tensor parallelism, Sec. 6.3):
+    statistics of one vocabulary shard [v_offset, v_offset + V_shard) per token: m = max_v z_v,
+    s = sum_v e^{z_v - m}, u = sum_v e^{z_v - m} z_v, the first global index of the maximum, and
+    z at the sampled token if the shard owns it (else -inf)."""
+    h, W_shard = _f64(h), _f64(W_shard)
+    y = np.asarray(y, dtype=np.int64)
+    Z = h @ W_shard.T
+    m = Z.max(axis=1)
+    E = np.exp(Z - m[:, None])
+    yl = y - v_offset
+    own = (yl >= 0) & (yl < W_shard.shape[0])
+    zy = np.full(len(y), -np.inf)
+    zy[own] = Z[np.flatnonzero(own), yl[own]]
+    return {"m": m, "s": E.sum(axis=1), "u": (E * Z).sum(axis=1),
+            "argmax": Z.argmax(axis=1) + v_offset, "zy": zy}
+
+
+def merge_shard_stats(stats):
+    """Combines the per-shard statistics of all shards (any partition of the vocabulary) into
+    lse, logp, entropy and argmax: M = max m_p, S = sum s_p e^{m_p - M}, U = sum u_p e^{m_p - M},
+    lse = M + log S, entropy = lse - U / S, logp = z_y - lse, argmax = lowest index attaining M."""
+    m = np.stack([st["m"] for st in stats])
+    M = m.max(axis=0)
+    sc = np.exp(m - M)
+    S_ = sum(st["s"] * sc[p] for p, st in enumerate(stats))
+    U = sum(st["u"] * sc[p] for p, st in enumerate(stats))
+    lse = M + np.log(S_)
+    zy = np.max(np.stack([st["zy"] for st in stats]), axis=0)
+    cand = np.stack([np.where(m[p] == M, st["argmax"], np.iinfo(np.int64).max)
+                     for p, st in enumerate(stats)])
+    return {"lse": lse, "logp": zy - lse, "entropy": lse - U / S_, "argmax": cand.min(axis=0)}
+
+
 def token_objective(logp, old, ref, adv_tok, eps_low, eps_high, beta):
     """Per-token GRPO terms (Sec. 6.1 clipped-ratio surrogate; Eq. 1 KL term with the
     per-token estimator) and their derivative with respect to logp.

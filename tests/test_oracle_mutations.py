@@ -36,6 +36,10 @@ MUTATIONS = [
     ("reward cap", "out[i] = min(10.0, t_base[i] / t_new[i] - 1.0)",
      "out[i] = min(10.0, t_base[i] / t_new[i])"),
     ("slower penalty", "out[i] = -1.0", "out[i] = -2.0"),
+    ("shard argmax keeps the highest index", "\"argmax\": cand.min(axis=0)}",
+     "\"argmax\": np.where(cand == np.iinfo(np.int64).max, -1, cand).max(axis=0)}"),
+    ("shard merge forgets the rescale", "U = sum(st[\"u\"] * sc[p] for p, st in enumerate(stats))",
+     "U = sum(st[\"u\"] for p, st in enumerate(stats))"),
     ("tool reward ratio inverted", "return lam * _f64(tools_used) / _f64(tools_avail)",
      "return lam * _f64(tools_avail) / _f64(tools_used)"),
 ]

@@ -332,11 +332,32 @@ def pin_golden_rewards(o):
         assert abs(r[0] - c["r"]) < 1e-12, c["why"]
 
 
+def pin_vocab_shards_merge_to_full_vocab(o):
+    """For any partition of the vocabulary into shards (uneven, tiny, with exact ties across
+    shards) the merged shard statistics equal the whole-vocabulary scoring."""
+    rng = np.random.default_rng(13)
+    n, d, V = 25, 12, 103
+    h = rng.normal(size=(n, d))
+    W = rng.normal(scale=0.4, size=(V, d))
+    a = int((h @ W.T).argmax(axis=1)[0])
+    b = (a + 51) % V
+    W[b] = W[a]                                      # exact tie for token 0, in another shard
+    cut = (min(a, b) + max(a, b)) // 2 + 1
+    y = rng.integers(0, V, size=n)
+    full = o.score_tokens(h, W, y)
+    for cuts in ([0, V], [0, 50, V], [0, 1, 40, 41, 90, V], [0, cut, V]):
+        st = [o.shard_stats(h, W[a:b], y, a) for a, b in zip(cuts[:-1], cuts[1:])]
+        mg = o.merge_shard_stats(st)
+        for k in ("lse", "logp", "entropy"):
+            np.testing.assert_allclose(mg[k], full[k], rtol=1e-12, atol=1e-12)
+        assert np.array_equal(mg["argmax"], full["argmax"])
+
+
 PINS = [pin_uniform_logits, pin_scipy_log_softmax, pin_scipy_entropy, pin_argmax_ties,
         pin_golden_objective, pin_golden_advantages, pin_advantages_scipy_and_invariants,
         pin_finite_differences, pin_on_policy_reinforce, pin_torch_autograd,
         pin_dW_rows_sum_to_zero, pin_vocab_row_subset, pin_counts, pin_sft_torch_cross_entropy,
-        pin_golden_rewards]
+        pin_golden_rewards, pin_vocab_shards_merge_to_full_vocab]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
