@@ -157,6 +157,47 @@ int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new
                  const int32_t* tools_used, const int32_t* tools_avail, int32_t n,
                  float lambda_tools, float* r_out, grpo_stream_t stream);
 
+/* Vocabulary-parallel (tensor-parallel) variant. The paper shards the policy over GPUs with
+ * tensor parallelism (Sec. 6.3); sharding the LM head by vocabulary rows needs one exchange of
+ * per-token statistics after the forward and one sum of dH after the backward.
+ *
+ * grpo_score_fwd_shard: this rank holds rows [v_offset, v_offset + V_shard) of W (W_shard
+ * [V_shard, d], bf16); tokens are global ids in [0, V_total). Writes, per position,
+ *   stats [S,T,4] f32: (m = max z, sum e^{z-m}, sum e^{z-m} z, argmax) over the shard, the
+ *                      argmax as the bit pattern of an int32 global index (16-byte aligned);
+ *   zy    [S,T] f32:   z at the sampled token if this shard owns it, else -inf.
+ * Unscored positions get (-inf, 0, 0, -1) and -inf. Workspace: grpo_workspace_bytes with
+ * V = V_shard. */
+int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
+                         const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                         int32_t d, int32_t V_shard, int32_t v_offset, int32_t V_total,
+                         float* stats, float* zy, void* workspace, size_t workspace_bytes,
+                         grpo_stream_t stream);
+
+/* Merges the statistics of all shards after they were exchanged (e.g. all-gathered so that
+ * stats is [num_shards, S, T, 4] and zy [num_shards, S, T]) into grpo_score_fwd's outputs:
+ * lse = M + log sum_p s_p e^{m_p - M}, logp = z_y - lse, entropy = lse - U/S, argmax = lowest
+ * global index attaining M; valid_count as in grpo_score_fwd. Needs 256 + 4*S bytes of
+ * workspace (rounded up to 256). */
+int grpo_merge_shard_stats(const float* stats, const float* zy, int32_t num_shards,
+                           const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                           int32_t V_total, float* logp, float* lse, float* entropy,
+                           int32_t* argmax, int32_t* valid_count, void* workspace,
+                           size_t workspace_bytes, grpo_stream_t stream);
+
+/* The shard's part of grpo_loss_bwd: logp/lse are the merged (global) values; the loss is the
+ * full loss (every rank computes it); dz is formed for this shard's columns only, so
+ * dH_partial [S,T,d] f32 is this shard's contribution (sum it over the ranks) and dW_shard
+ * [V_shard, d] f32 is this shard's rows of dW. bf16 only. */
+int grpo_loss_bwd_shard(const void* H, const void* W_shard, int32_t dtype,
+                        const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                        int32_t d, int32_t V_shard, int32_t v_offset, int32_t V_total,
+                        const float* logp, const float* lse, const float* old_logp,
+                        const float* ref_logp, const float* adv, const int32_t* valid_count,
+                        float eps_low, float eps_high, float beta, int32_t agg, double norm,
+                        float* loss_out, float* dH_partial, float* dW_shard, void* workspace,
+                        size_t workspace_bytes, grpo_stream_t stream);
+
 /* Synchronises `stream`, returns the first device-side status recorded in the workspace since
  * the last call (GRPO_OK if none) and clears it. *where_out (may be NULL) gets a code naming the
  * kernel and wait that recorded it. */
@@ -171,7 +212,7 @@ enum {
   GRPO_K_MASK_SCAN = 0, GRPO_K_TILE_LIST, GRPO_K_GROUP_ADV, GRPO_K_FWD_GEMM, GRPO_K_FWD_MERGE,
   GRPO_K_LOSS_TOKENS, GRPO_K_LOSS_FINAL, GRPO_K_BWD_DZ_GEMM, GRPO_K_BWD_DH_GEMM,
   GRPO_K_BWD_DW_GEMM, GRPO_K_DH_ZERO_TAIL, GRPO_K_F32_FWD, GRPO_K_F32_DH, GRPO_K_F32_DW,
-  GRPO_K_REWARDS, GRPO_K_COUNT
+  GRPO_K_REWARDS, GRPO_K_SHARD_STATS, GRPO_K_MERGE_SHARDS, GRPO_K_COUNT
 };
 const char* grpo_kernel_name(int32_t kernel_id);
 int grpo_timing_enable(int32_t enable);   /* 1 = record events from now on, 0 = stop */

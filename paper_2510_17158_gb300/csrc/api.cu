@@ -21,7 +21,8 @@ namespace {
 const char* const kKernelNames[GRPO_K_COUNT] = {
     "mask_scan",       "tile_list",    "group_adv",   "fwd_gemm_tc",  "fwd_merge",
     "loss_tokens",     "loss_final",   "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw",      "rewards"};
+    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw",      "rewards",
+    "shard_stats",     "merge_shards"};
 
 struct EventPair {
   cudaEvent_t a, b;
@@ -352,7 +353,7 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
                   const float* ref_logp, const float* adv, const int32_t* valid_count,
                   float eps_low, float eps_high, float beta, int32_t agg, double norm,
                   float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
-                  grpo_stream_t stream) {
+                  grpo_stream_t stream, int32_t v_offset = 0, bool dh_f32 = false) {
   if (!H || !W || !tokens || !mask || !logp || !lse || !valid_count || !loss_out || !dH || !dW)
     return GRPO_ERR_INVALID_ARG;
   if (mode == 0 && (!old_logp || !adv)) return GRPO_ERR_INVALID_ARG;
@@ -438,6 +439,8 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     return GRPO_ERR_CUDA;
 
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
+  a.v_offset = v_offset;
+  a.dh_f32 = dh_f32 ? 1 : 0;
   a.g = v.g;
   a.lse = lse;
   a.dz = dz;
@@ -463,7 +466,7 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     }));
   }
   return counted(GRPO_K_DH_ZERO_TAIL, st, [&] {
-    return launch_dh_zero_tail(v.seq_tile_base, S, T, d, static_cast<__nv_bfloat16*>(dH), st);
+    return launch_dh_zero_tail(v.seq_tile_base, S, T, d, dH, dh_f32 ? 4 : 2, st);
   });
 }
 
@@ -491,6 +494,90 @@ int grpo_sft_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t
   return loss_bwd_impl(1, H, W, dtype, tokens, mask, S, T, d, V, logp, lse, nullptr, nullptr,
                        nullptr, valid_count, 0.f, 0.f, 0.f, agg, norm, loss_out, dH, dW, workspace,
                        workspace_bytes, stream);
+}
+
+int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
+                         const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                         int32_t d, int32_t V_shard, int32_t v_offset, int32_t V_total,
+                         float* stats, float* zy, void* workspace, size_t workspace_bytes,
+                         grpo_stream_t stream) {
+  if (!H || !W_shard || !tokens || !mask || !stats || !zy) return GRPO_ERR_INVALID_ARG;
+  if (!shape_ok(S, T, d, V_shard) || v_offset < 0 || V_total <= 0 ||
+      static_cast<long long>(v_offset) + V_shard > V_total)
+    return GRPO_ERR_INVALID_ARG;
+  if (dtype != GRPO_BF16) return GRPO_ERR_UNSUPPORTED;
+  GRPO_TRY(check_dtype_shape(dtype, d));
+  if (!aligned16(H) || !aligned16(W_shard) || !aligned16(stats)) return GRPO_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
+  const Layout L = make_layout(S, T, d, V_shard, dtype);
+  if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const Views v = views(workspace, L);
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, v.counts, v.seq_last, st); }));
+  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
+    return launch_tile_list(v.seq_last, v.counts, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
+  }));
+  const bool pair = g_cta_pair.load() != 0;
+  CUtensorMap mapH, mapW;
+  if (!make_map(&mapH, H, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+      !make_map(&mapW, W_shard, d, V_shard, d, pair ? kTileN / 2 : kTileN))
+    return GRPO_ERR_CUDA;
+  GemmArgs a = base_args(L, v, S, T, d, V_shard, tokens, mask);
+  a.v_offset = v_offset;
+  a.partials = v.partials;
+  a.zy = v.zy;
+  GRPO_TRY(counted(GRPO_K_FWD_GEMM, st, [&] {
+    return launch_gemm(ROLE_FWD, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, pair), pair,
+                       st);
+  }));
+  return counted(GRPO_K_SHARD_STATS, st, [&] {
+    return launch_shard_stats(v.partials, L.rows_cap, L.num_strips, v.zy, v.seq_tile_base, tokens,
+                              mask, S, T, V_shard, v_offset, reinterpret_cast<float4*>(stats), zy,
+                              st);
+  });
+}
+
+int grpo_merge_shard_stats(const float* stats, const float* zy, int32_t num_shards,
+                           const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                           int32_t V_total, float* logp, float* lse, float* entropy,
+                           int32_t* argmax, int32_t* valid_count, void* workspace,
+                           size_t workspace_bytes, grpo_stream_t stream) {
+  if (!stats || !zy || !tokens || !mask || !logp || !lse || !entropy || !argmax || !valid_count)
+    return GRPO_ERR_INVALID_ARG;
+  if (num_shards <= 0 || S <= 0 || T <= 0 || V_total <= 0 ||
+      static_cast<long long>(S) * T >= (1ll << 31))
+    return GRPO_ERR_INVALID_ARG;
+  if (!aligned16(stats)) return GRPO_ERR_INVALID_ARG;
+  if (!workspace || workspace_bytes < sizeof(WsHeader) + align256(sizeof(int32_t) * S) ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  WsHeader* hdr = static_cast<WsHeader*>(workspace);
+  int32_t* seq_last = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) + sizeof(WsHeader));
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, valid_count, seq_last, st); }));
+  return counted(GRPO_K_MERGE_SHARDS, st, [&] {
+    return launch_merge_shards(reinterpret_cast<const float4*>(stats), zy, num_shards, tokens,
+                               mask, S, T, V_total, logp, lse, entropy, argmax, hdr, st);
+  });
+}
+
+int grpo_loss_bwd_shard(const void* H, const void* W_shard, int32_t dtype,
+                        const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
+                        int32_t d, int32_t V_shard, int32_t v_offset, int32_t V_total,
+                        const float* logp, const float* lse, const float* old_logp,
+                        const float* ref_logp, const float* adv, const int32_t* valid_count,
+                        float eps_low, float eps_high, float beta, int32_t agg, double norm,
+                        float* loss_out, float* dH_partial, float* dW_shard, void* workspace,
+                        size_t workspace_bytes, grpo_stream_t stream) {
+  if (v_offset < 0 || V_total <= 0 || V_shard <= 0 ||
+      static_cast<long long>(v_offset) + V_shard > V_total)
+    return GRPO_ERR_INVALID_ARG;
+  if (dtype != GRPO_BF16) return GRPO_ERR_UNSUPPORTED;
+  return loss_bwd_impl(0, H, W_shard, dtype, tokens, mask, S, T, d, V_shard, logp, lse, old_logp,
+                       ref_logp, adv, valid_count, eps_low, eps_high, beta, agg, norm, loss_out,
+                       dH_partial, dW_shard, workspace, workspace_bytes, stream, v_offset, true);
 }
 
 int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new,

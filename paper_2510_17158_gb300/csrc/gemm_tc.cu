@@ -346,7 +346,8 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       const int2 tl = a.tiles[m_load];
       const bool rv = m_ok && tl.y + r < a.T;
       const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
-      const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] : -1;
+      // sampled token as a column of this W (a vocabulary shard's rows start at v_offset)
+      const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] - a.v_offset : -1;
       float rm = -INFINITY, rs = 0.f, ru = 0.f, zyv = 0.f;
       int ri = 0;
       bool found = false;
@@ -418,7 +419,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       const bool act = rv && a.mask[pos] != 0;
       const float gt = act ? a.g[pos] : 0.f;
       const float ll = act ? a.lse[pos] * kLog2e : 0.f;
-      const int y = act ? a.tokens[pos] : -1;
+      const int y = act ? a.tokens[pos] - a.v_offset : -1;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
       __nv_bfloat16* dst_row =
@@ -480,6 +481,11 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
           for (int j = 0; j < 8; ++j)
             reinterpret_cast<float4*>(acc_row)[j] =
                 make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
+        } else if (a.dh_f32) {
+          float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(a.dH) + pos * a.d + col);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
         } else {
           uint4* dst = reinterpret_cast<uint4*>(a.dH + pos * a.d + col);
 #pragma unroll

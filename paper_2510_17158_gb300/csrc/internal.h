@@ -49,6 +49,10 @@ struct GemmArgs {
   float* dW;
   // test hook: nonzero makes CTA 0's producer leave its first stage unfilled
   int inject_stall;
+  // vocabulary-parallel shard: W holds global rows v_offset .. v_offset + V - 1 (0 otherwise)
+  int v_offset;
+  // DH: write the final dH in f32 (a shard's partial sum) instead of H's dtype
+  int dh_f32;
 };
 
 // Launches (all asynchronous on `st`; return the cudaError_t of the launch).
@@ -74,8 +78,17 @@ cudaError_t launch_rewards(const uint8_t* correct, const float* t_base, const fl
                            float* r, cudaStream_t st);
 cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm,
                               const WsHeader* hdr, float* loss_out, cudaStream_t st);
-cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d,
-                                __nv_bfloat16* dH, cudaStream_t st);
+cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d, void* dH,
+                                int elem_bytes, cudaStream_t st);
+cudaError_t launch_shard_stats(const float4* partials, long long rows_cap, int num_strips,
+                               const float* zy_ws, const int32_t* seq_tile_base,
+                               const int32_t* tokens, const uint8_t* mask, int S, int T,
+                               int V_shard, int v_offset, float4* stats, float* zy_out,
+                               cudaStream_t st);
+cudaError_t launch_merge_shards(const float4* stats, const float* zy, int P,
+                                const int32_t* tokens, const uint8_t* mask, int S, int T,
+                                int V_total, float* logp, float* lse, float* entropy,
+                                int32_t* argmax, WsHeader* hdr, cudaStream_t st);
 cudaError_t launch_f32_fwd(const float* H, const float* W, const int32_t* tokens,
                            const uint8_t* mask, int S, int T, int d, int V, float* logp,
                            float* lse, float* entropy, int32_t* argmax, WsHeader* hdr,

@@ -323,18 +323,107 @@ __global__ void k_loss_final(const float* __restrict__ seq_loss, int S, float* l
 // dH rows that no token tile covers (positions after a sequence's last tile) are zero.
 // ------------------------------------------------------------------------------------------
 __global__ void k_dh_zero_tail(const int32_t* __restrict__ seq_tile_base, int S, int T, int d,
-                               __nv_bfloat16* __restrict__ dH) {
+                               char* __restrict__ dH, int elem_bytes) {
   const int tb = blockIdx.x, i = blockIdx.y;
   const int covered = seq_tile_base[i + 1] - seq_tile_base[i];
   if (tb < covered) return;
   const int t0 = tb * kTileRows;
   const int t1 = min(T, t0 + kTileRows);
   if (t0 >= t1) return;
-  const size_t beg = (static_cast<size_t>(i) * T + t0) * d;
-  const size_t n = static_cast<size_t>(t1 - t0) * d;   // multiple of 8 (d % 64 == 0)
+  const size_t beg = (static_cast<size_t>(i) * T + t0) * d * elem_bytes;
+  const size_t n = static_cast<size_t>(t1 - t0) * d * elem_bytes / 2;  // d % 64 == 0
   uint4* p = reinterpret_cast<uint4*>(dH + beg);
   const uint4 z = make_uint4(0, 0, 0, 0);
   for (size_t k = threadIdx.x; k < n / 8; k += blockDim.x) p[k] = z;
+}
+
+// ------------------------------------------------------------------------------------------
+// Vocabulary-parallel scoring: statistics of one shard per position, and the merge of the
+// statistics of all shards.
+// ------------------------------------------------------------------------------------------
+__global__ void k_shard_stats(const float4* __restrict__ partials, long long rows_cap,
+                              int num_strips, const float* __restrict__ zy_ws,
+                              const int32_t* __restrict__ seq_tile_base,
+                              const int32_t* __restrict__ tokens,
+                              const uint8_t* __restrict__ mask, int S, int T, int V_shard,
+                              int v_offset, float4* __restrict__ stats,
+                              float* __restrict__ zy_out) {
+  const long long pos = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (pos >= static_cast<long long>(S) * T) return;
+  if (mask[pos] == 0) {
+    stats[pos] = make_float4(-INFINITY, 0.f, 0.f, __int_as_float(-1));
+    zy_out[pos] = -INFINITY;
+    return;
+  }
+  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
+  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
+                        (t % kTileRows);
+  float M = -INFINITY;
+  int idx = 0;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    if (p.x > M) {
+      M = p.x;
+      idx = __float_as_int(p.w);
+    }
+  }
+  float Ssum = 0.f, U = 0.f;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    const float sc = ex2_approx((p.x - M) * kLog2e);
+    Ssum = fmaf(p.y, sc, Ssum);
+    U = fmaf(p.z, sc, U);
+  }
+  stats[pos] = make_float4(M, Ssum, U, __int_as_float(idx + v_offset));
+  const int yl = tokens[pos] - v_offset;
+  zy_out[pos] = (yl >= 0 && yl < V_shard) ? zy_ws[pos] : -INFINITY;
+}
+
+__global__ void k_merge_shards(const float4* __restrict__ stats, const float* __restrict__ zy,
+                               int P, const int32_t* __restrict__ tokens,
+                               const uint8_t* __restrict__ mask, int S, int T, int V_total,
+                               float* __restrict__ logp, float* __restrict__ lse_out,
+                               float* __restrict__ entropy, int32_t* __restrict__ argmax,
+                               WsHeader* hdr) {
+  const long long n = static_cast<long long>(S) * T;
+  const long long pos = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (pos >= n) return;
+  if (mask[pos] == 0) {
+    logp[pos] = 0.f;
+    lse_out[pos] = 0.f;
+    entropy[pos] = 0.f;
+    argmax[pos] = -1;
+    return;
+  }
+  float M = -INFINITY, zyv = -INFINITY;
+  int idx = 0x7fffffff;
+  for (int p = 0; p < P; ++p) {
+    const float4 s = stats[p * n + pos];
+    const int ip = __float_as_int(s.w);
+    if (s.x > M || (s.x == M && ip < idx)) {  // lowest global index among the maxima
+      M = s.x;
+      idx = ip;
+    }
+    zyv = fmaxf(zyv, zy[p * n + pos]);
+  }
+  float Ssum = 0.f, U = 0.f;
+  for (int p = 0; p < P; ++p) {
+    const float4 s = stats[p * n + pos];
+    const float sc = ex2_approx((s.x - M) * kLog2e);
+    Ssum = fmaf(s.y, sc, Ssum);
+    U = fmaf(s.z, sc, U);
+  }
+  const float lse = M + logf(Ssum);
+  const int y = tokens[pos];
+  float lp = zyv - lse;
+  if (y < 0 || y >= V_total) {
+    record_error(hdr, ST_TOKEN_RANGE, WHERE_MERGE_TOKEN);
+    lp = __int_as_float(0x7fc00000);
+  }
+  logp[pos] = lp;
+  lse_out[pos] = lse;
+  entropy[pos] = lse - U / Ssum;
+  argmax[pos] = idx;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -590,10 +679,33 @@ cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm
   return cudaGetLastError();
 }
 
-cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d,
-                                __nv_bfloat16* dH, cudaStream_t st) {
+cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d, void* dH,
+                                int elem_bytes, cudaStream_t st) {
   dim3 grid((T + kTileRows - 1) / kTileRows, S);
-  k_dh_zero_tail<<<grid, 256, 0, st>>>(seq_tile_base, S, T, d, dH);
+  k_dh_zero_tail<<<grid, 256, 0, st>>>(seq_tile_base, S, T, d, static_cast<char*>(dH),
+                                       elem_bytes);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_shard_stats(const float4* partials, long long rows_cap, int num_strips,
+                               const float* zy_ws, const int32_t* seq_tile_base,
+                               const int32_t* tokens, const uint8_t* mask, int S, int T,
+                               int V_shard, int v_offset, float4* stats, float* zy_out,
+                               cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  k_shard_stats<<<static_cast<unsigned>((P + 255) / 256), 256, 0, st>>>(
+      partials, rows_cap, num_strips, zy_ws, seq_tile_base, tokens, mask, S, T, V_shard,
+      v_offset, stats, zy_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_shards(const float4* stats, const float* zy, int P,
+                                const int32_t* tokens, const uint8_t* mask, int S, int T,
+                                int V_total, float* logp, float* lse, float* entropy,
+                                int32_t* argmax, WsHeader* hdr, cudaStream_t st) {
+  const long long n = static_cast<long long>(S) * T;
+  k_merge_shards<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(
+      stats, zy, P, tokens, mask, S, T, V_total, logp, lse, entropy, argmax, hdr);
   return cudaGetLastError();
 }
 

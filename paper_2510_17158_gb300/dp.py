@@ -1,4 +1,5 @@
-"""Host-side data-parallel sharding of a GRPO batch over ranks (whole groups per rank).
+"""Host-side sharding of a GRPO batch over ranks: data-parallel (whole groups per rank) and
+vocabulary-parallel (rows of the LM head per rank).
 
 Advantages are normalised within a group (Alg. 1), so a rank must own whole groups; the loss
 normaliser of Eq. 1's expectation must be the global one (S' sequences for seq_mean, N' scored
@@ -31,3 +32,12 @@ def global_norm(agg: str, local_seqs: int, local_tokens: int, all_reduce_sum) ->
     if agg == "token_mean":
         return float(all_reduce_sum(float(local_tokens)))
     raise ValueError(agg)
+
+
+def vocab_shard_bounds(V: int, world_size: int, rank: int, align: int = 256):
+    """Rows [v0, v1) of the LM head held by `rank` when the vocabulary is split over
+    `world_size` ranks in blocks aligned to `align` rows (the last shard takes the remainder)."""
+    blocks = (V + align - 1) // align
+    b0 = (blocks * rank) // world_size
+    b1 = (blocks * (rank + 1)) // world_size
+    return min(V, b0 * align), min(V, b1 * align)

@@ -27,7 +27,8 @@ STATUS_NAMES = {0: "GRPO_OK", -1: "GRPO_ERR_INVALID_ARG", -2: "GRPO_ERR_UNSUPPOR
                 -6: "GRPO_ERR_TIMEOUT", -7: "GRPO_ERR_GROUPS"}
 KERNEL_NAMES = ["mask_scan", "tile_list", "group_adv", "fwd_gemm_tc", "fwd_merge", "loss_tokens",
                 "loss_final", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-                "dh_zero_tail", "f32_fwd", "f32_dh", "f32_dw", "rewards"]
+                "dh_zero_tail", "f32_fwd", "f32_dh", "f32_dw", "rewards", "shard_stats",
+                "merge_shards"]
 
 
 class GrpoError(RuntimeError):
@@ -63,6 +64,13 @@ def _declare(lib):
         "grpo_sft_loss_bwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                              _p, _p, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
         "grpo_rewards": (ctypes.c_int, [_p, _p, _p, _p, _p, _i32, _f32, _p, _p]),
+        "grpo_score_fwd_shard": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32,
+                                                _i32, _i32, _p, _p, _p, _sz, _p]),
+        "grpo_merge_shard_stats": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _p, _p,
+                                                  _p, _p, _p, _p, _sz, _p]),
+        "grpo_loss_bwd_shard": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32,
+                                               _i32, _i32, _p, _p, _p, _p, _p, _p, _f32, _f32,
+                                               _f32, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
         "grpo_score_fwd_static": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                                  _p, _p, _p, _p, _p, _p]),
     }
@@ -311,6 +319,68 @@ def grpo_rewards(correct, t_base, t_new, tools_used, tools_avail, lambda_tools=0
                              _stream(stream))
     _check(st, "grpo_rewards")
     return r_out
+
+
+def grpo_score_fwd_shard(H, W_shard, tokens, mask, v_offset: int, V_total: int, ws: Workspace,
+                         out: Optional[dict] = None, stream=None) -> dict:
+    """Statistics of one vocabulary shard: dict(stats [S,T,4] f32, zy [S,T] f32)."""
+    S, T, d = H.shape
+    Vs = W_shard.shape[0]
+    _need(H, "H", torch.bfloat16)
+    _need(W_shard, "W_shard", torch.bfloat16, (Vs, d))
+    _need(tokens, "tokens", torch.int32, (S, T))
+    _need(mask, "mask", torch.uint8, (S, T))
+    if out is None:
+        out = {"stats": torch.empty((S, T, 4), dtype=torch.float32, device=H.device),
+               "zy": torch.empty((S, T), dtype=torch.float32, device=H.device)}
+    st = _lib().grpo_score_fwd_shard(_ptr(H), _ptr(W_shard), GRPO_BF16, _ptr(tokens), _ptr(mask),
+                                     S, T, d, Vs, int(v_offset), int(V_total), _ptr(out["stats"]),
+                                     _ptr(out["zy"]), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "grpo_score_fwd_shard")
+    return out
+
+
+def grpo_merge_shard_stats(stats, zy, tokens, mask, V_total: int, ws: Workspace,
+                           out: Optional[dict] = None, stream=None) -> dict:
+    """Merge of stacked shard statistics (stats [P,S,T,4], zy [P,S,T]) into the forward outputs."""
+    P, S, T = zy.shape
+    _need(stats, "stats", torch.float32, (P, S, T, 4))
+    _need(zy, "zy", torch.float32, (P, S, T))
+    if out is None:
+        f = dict(dtype=torch.float32, device=zy.device)
+        out = {"logp": torch.empty((S, T), **f), "lse": torch.empty((S, T), **f),
+               "entropy": torch.empty((S, T), **f),
+               "argmax": torch.empty((S, T), dtype=torch.int32, device=zy.device),
+               "valid_count": torch.empty((S,), dtype=torch.int32, device=zy.device)}
+    st = _lib().grpo_merge_shard_stats(_ptr(stats), _ptr(zy), P, _ptr(tokens), _ptr(mask), S, T,
+                                       int(V_total), _ptr(out["logp"]), _ptr(out["lse"]),
+                                       _ptr(out["entropy"]), _ptr(out["argmax"]),
+                                       _ptr(out["valid_count"]), ws.ptr, ws.nbytes,
+                                       _stream(stream))
+    _check(st, "grpo_merge_shard_stats")
+    return out
+
+
+def grpo_loss_bwd_shard(H, W_shard, tokens, mask, v_offset: int, V_total: int, logp, lse,
+                        old_logp, ref_logp, adv, valid_count, ws: Workspace, eps_low=0.2,
+                        eps_high=0.2, beta=0.04, agg="seq_mean", norm=0.0,
+                        out: Optional[dict] = None, stream=None) -> dict:
+    """The shard's backward: dict(loss [1], dH_partial [S,T,d] f32, dW_shard [V_shard,d] f32)."""
+    S, T, d = H.shape
+    Vs = W_shard.shape[0]
+    if out is None:
+        out = {"loss": torch.empty((1,), dtype=torch.float32, device=H.device),
+               "dH_partial": torch.empty((S, T, d), dtype=torch.float32, device=H.device),
+               "dW_shard": torch.empty((Vs, d), dtype=torch.float32, device=H.device)}
+    st = _lib().grpo_loss_bwd_shard(_ptr(H), _ptr(W_shard), GRPO_BF16, _ptr(tokens), _ptr(mask),
+                                    S, T, d, Vs, int(v_offset), int(V_total), _ptr(logp),
+                                    _ptr(lse), _ptr(old_logp), _ptr(ref_logp), _ptr(adv),
+                                    _ptr(valid_count), float(eps_low), float(eps_high),
+                                    float(beta), AGG_MODES[agg], float(norm), _ptr(out["loss"]),
+                                    _ptr(out["dH_partial"]), _ptr(out["dW_shard"]), ws.ptr,
+                                    ws.nbytes, _stream(stream))
+    _check(st, "grpo_loss_bwd_shard")
+    return out
 
 
 def grpo_last_device_error(ws: Workspace, stream=None):
