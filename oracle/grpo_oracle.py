@@ -141,6 +141,30 @@ def merge_shard_stats(stats):
     return {"lse": lse, "logp": zy - lse, "entropy": lse - U / S_, "argmax": cand.min(axis=0)}
 
 
+def exact_kl(h, W, h_ref, W_ref):
+    """Eq. 1's KL(pi_theta(.|c) || pi_ref(.|c)) at each scored position, over the whole
+    vocabulary: KL_t = sum_v p_tv (log p_tv - log q_tv), p = softmax(W h_t) (policy),
+    q = softmax(W_ref h_ref_t) (the frozen reference model of Alg. 1, its own hidden state and
+    LM head). The KL of the completion is the sum of KL_t over its tokens (chain rule)."""
+    Z = _f64(h) @ _f64(W).T
+    Zr = _f64(h_ref) @ _f64(W_ref).T
+    lse = Z.max(axis=1) + np.log(np.exp(Z - Z.max(axis=1)[:, None]).sum(axis=1))
+    lser = Zr.max(axis=1) + np.log(np.exp(Zr - Zr.max(axis=1)[:, None]).sum(axis=1))
+    logP = Z - lse[:, None]
+    logQ = Zr - lser[:, None]
+    P = np.exp(logP)
+    return {"kl": (P * (logP - logQ)).sum(axis=1), "lse_ref": lser, "logP": logP, "logQ": logQ}
+
+
+def exact_kl_logit_grads(h, W, y, lse, g, h_ref, W_ref, c):
+    """dL/dz_t for a loss sum_t [g-weighted log-prob term + c_t KL_t]: g_t (onehot(y_t) - p_t)
+    + c_t p_t (log p_t - log q_t - KL_t), the second term being d KL_t / d z_t."""
+    ek = exact_kl(h, W, h_ref, W_ref)
+    P = np.exp(ek["logP"])
+    dZ = logit_grads(h, W, y, lse, g)
+    return dZ + _f64(c)[:, None] * P * (ek["logP"] - ek["logQ"] - ek["kl"][:, None])
+
+
 def token_objective(logp, old, ref, adv_tok, eps_low, eps_high, beta):
     """Per-token GRPO terms (Sec. 6.1 clipped-ratio surrogate; Eq. 1 KL term with the
     per-token estimator) and their derivative with respect to logp.
@@ -269,6 +293,42 @@ def sft_step(H, W, tokens, mask, agg=TOKEN_MEAN, norm=None, vocab_rows=None, wit
         dH[si, ti] = dHv
         out["dH"] = dH
         out["dW"] = dW
+    return out
+
+
+def grpo_step_exact_kl(H, W, H_ref, W_ref, tokens, mask, rewards, group_offsets, old,
+                       eps_low=0.2, eps_high=0.2, beta=0.04, agg=SEQ_MEAN, std_mode="unbiased",
+                       std_eps=1e-4, norm=None, with_grads=True):
+    """GRPO with Eq. 1's KL term taken exactly over the vocabulary: l_t = -surr_t + beta KL_t;
+    dH, dW through dz = g (onehot - p) + beta w p (log p - log q - KL)."""
+    H = _f64(H)
+    S, T, d = H.shape
+    mask = np.asarray(mask)
+    counts = valid_counts(mask)
+    adv = group_advantages(rewards, group_offsets, std_mode, std_eps)
+    idx = np.argwhere(mask != 0)
+    si, ti = idx[:, 0], idx[:, 1]
+    h, hr = H[si, ti], _f64(H_ref)[si, ti]
+    y = np.asarray(tokens)[si, ti]
+    sc = score_tokens(h, W, y)
+    ek = exact_kl(h, W, hr, W_ref)
+    tob = token_objective(sc["logp"], _f64(old)[si, ti], sc["logp"], adv[si], eps_low, eps_high,
+                          0.0)
+    ell = tob["ell"] + beta * ek["kl"]
+    L, g_tok, mass = aggregate(ell, tob["dell"], si, counts, S, agg, norm)
+    _, w_tok, _ = aggregate(np.zeros_like(ell), np.ones_like(ell), si, counts, S, agg, norm)
+    out = {"counts": counts, "adv": adv, "loss": L, "loss_abs_mass": mass}
+    for k, v in (("logp", sc["logp"]), ("lse", sc["lse"]), ("kl", ek["kl"]),
+                 ("lse_ref", ek["lse_ref"]), ("entropy", sc["entropy"])):
+        a = np.zeros((S, T))
+        a[si, ti] = v
+        out[k] = a
+    if with_grads:
+        dZ = exact_kl_logit_grads(h, W, y, sc["lse"], g_tok, hr, W_ref, beta * w_tok)
+        dH = np.zeros((S, T, d))
+        dH[si, ti] = dZ @ _f64(W)
+        out["dH"] = dH
+        out["dW"] = dZ.T @ h
     return out
 
 

@@ -40,6 +40,10 @@ MUTATIONS = [
      "\"argmax\": np.where(cand == np.iinfo(np.int64).max, -1, cand).max(axis=0)}"),
     ("shard merge forgets the rescale", "U = sum(st[\"u\"] * sc[p] for p, st in enumerate(stats))",
      "U = sum(st[\"u\"] for p, st in enumerate(stats))"),
+    ("exact-KL gradient drops -KL", "* P * (ek[\"logP\"] - ek[\"logQ\"] - ek[\"kl\"][:, None])",
+     "* P * (ek[\"logP\"] - ek[\"logQ\"])"),
+    ("exact KL reversed", "\"kl\": (P * (logP - logQ)).sum(axis=1)",
+     "\"kl\": (np.exp(logQ) * (logQ - logP)).sum(axis=1)"),
     ("tool reward ratio inverted", "return lam * _f64(tools_used) / _f64(tools_avail)",
      "return lam * _f64(tools_avail) / _f64(tools_used)"),
 ]

@@ -353,11 +353,59 @@ def pin_vocab_shards_merge_to_full_vocab(o):
         assert np.array_equal(mg["argmax"], full["argmax"])
 
 
+def pin_exact_kl_torch_and_finite_differences(o):
+    """The exact per-token KL equals torch.distributions.kl_divergence of the two categorical
+    distributions, is 0 when the reference equals the policy, and the GRPO loss with the exact
+    KL has dH / dW equal to central finite differences (V = 9, d = 5)."""
+    rng = np.random.default_rng(17)
+    n, d, V = 7, 5, 9
+    h, hr = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    W, Wr = rng.normal(scale=0.6, size=(V, d)), rng.normal(scale=0.6, size=(V, d))
+    ek = o.exact_kl(h, W, hr, Wr)
+    tk = torch.distributions.kl_divergence(
+        torch.distributions.Categorical(logits=torch.tensor(h @ W.T)),
+        torch.distributions.Categorical(logits=torch.tensor(hr @ Wr.T))).numpy()
+    np.testing.assert_allclose(ek["kl"], tk, rtol=1e-10, atol=1e-13)
+    assert np.all(ek["kl"] >= 0)
+    np.testing.assert_allclose(o.exact_kl(h, W, h, W)["kl"], 0.0, atol=1e-13)
+    S, T = 2, 4
+    H = rng.normal(size=(S, T, d))
+    Hr = rng.normal(size=(S, T, d))
+    mask = np.ones((S, T), np.uint8)
+    mask[1, 3] = 0
+    tok = rng.integers(0, V, size=(S, T))
+    rew = np.array([0.3, 1.1], np.float32)
+    go = np.array([0, 2])
+    old = rng.normal(-2.2, 0.7, size=(S, T))
+    beta = 0.3
+    base = o.grpo_step_exact_kl(H, W, Hr, Wr, tok, mask, rew, go, old, 0.2, 0.2, beta)
+    step = 1e-6
+
+    def L_of(Hx, Wx):
+        return o.grpo_step_exact_kl(Hx, Wx, Hr, Wr, tok, mask, rew, go, old, 0.2, 0.2, beta,
+                                    with_grads=False)["loss"]
+    for idx in np.ndindex(*H.shape):
+        if not mask[idx[0], idx[1]]:
+            continue
+        Hp, Hm = H.copy(), H.copy()
+        Hp[idx] += step
+        Hm[idx] -= step
+        num = (L_of(Hp, W) - L_of(Hm, W)) / (2 * step)
+        assert abs(num - base["dH"][idx]) <= 1e-6 * max(1e-3, abs(num)), (idx, num, base["dH"][idx])
+    for idx in np.ndindex(*W.shape):
+        Wp, Wm = W.copy(), W.copy()
+        Wp[idx] += step
+        Wm[idx] -= step
+        num = (L_of(H, Wp) - L_of(H, Wm)) / (2 * step)
+        assert abs(num - base["dW"][idx]) <= 1e-6 * max(1e-3, abs(num)), (idx, num, base["dW"][idx])
+
+
 PINS = [pin_uniform_logits, pin_scipy_log_softmax, pin_scipy_entropy, pin_argmax_ties,
         pin_golden_objective, pin_golden_advantages, pin_advantages_scipy_and_invariants,
         pin_finite_differences, pin_on_policy_reinforce, pin_torch_autograd,
         pin_dW_rows_sum_to_zero, pin_vocab_row_subset, pin_counts, pin_sft_torch_cross_entropy,
-        pin_golden_rewards, pin_vocab_shards_merge_to_full_vocab]
+        pin_golden_rewards, pin_vocab_shards_merge_to_full_vocab,
+        pin_exact_kl_torch_and_finite_differences]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
