@@ -243,6 +243,11 @@ def run_gpu(args):
     old = (f0["logp"] + b.noise_old).contiguous()
     ref = (f0["logp"] + b.noise_ref).contiguous()
     fwd_out = {k: torch.empty_like(v) for k, v in f0.items()}
+    if args.path == "grpo-exact-kl":
+        from paper_2510_17158_gb300.synthetic import reference_model_inputs
+        H_ref, W_ref = reference_model_inputs(b)
+        fwd_out["lse_ref"] = torch.empty_like(f0["lse"])
+        fwd_out["kl"] = torch.empty_like(f0["lse"])
     bwd_out = {"loss": torch.empty(1, device=device), "dH": torch.empty_like(b.H),
                "dW": torch.empty((V, d), dtype=torch.float32, device=device)}
     adv = torch.empty(S, device=device)
@@ -250,6 +255,11 @@ def run_gpu(args):
     gen_s = time.time() - t_gen
 
     def step(H, W, tok, mask, rewards, go, old_, ref_):
+        if args.path == "grpo-exact-kl":   # Eq. 1's KL over the whole vocabulary
+            G.group_advantages(rewards, go, ws, adv_out=adv)
+            f = G.grpo_score_fwd_kl(H, W, H_ref, W_ref, tok, mask, ws, out=fwd_out)
+            return G.grpo_loss_bwd_kl(H, W, H_ref, W_ref, tok, mask, f, old_, adv, ws,
+                                      eps_low=w.eps, eps_high=w.eps, beta=w.beta, out=bwd_out)
         if args.path == "sft":       # distillation step (Sec. 6.2): no advantages, no ratio
             f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
             return G.grpo_sft_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], f["valid_count"],
@@ -314,7 +324,10 @@ def run_gpu(args):
     e2e_value = total_tokens * e2e_steps / e2e_s
     pk = peaks()
     step_ms = ms_max / args.steps
-    alg_tflops = lm_head_flops(N_v, d, V) / (step_ms / 1e3) / 1e12
+    # algorithmic flop per step: 6 N d V (fwd, dH, dW); the exact-KL path adds the reference
+    # model's forward product (8 N d V). Recomputed products count as overhead, not work.
+    alg_flop = lm_head_flops(N_v, d, V) * (8.0 / 6.0 if args.path == "grpo-exact-kl" else 1.0)
+    alg_tflops = alg_flop / (step_ms / 1e3) / 1e12
 
     # ---- roofline of the dominant kernel -------------------------------------------------------
     per_kernel = {k: {"launches": n, "ms_total": round(t, 3), "ms_per_launch": round(t / n, 4),
@@ -322,8 +335,9 @@ def run_gpu(args):
     dom = max(table, key=lambda k: table[k][1])
     n_dom, t_dom = table[dom]
     chunk = args.vocab_chunk or V
+    kl2 = 2.0 if args.path == "grpo-exact-kl" else 1.0
     flops_per_launch = {
-        "fwd_gemm_tc": 2.0 * N_v * d * V, "bwd_dz_gemm_tc": 2.0 * N_v * d * min(V, chunk),
+        "fwd_gemm_tc": 2.0 * kl2 * N_v * d * V, "bwd_dz_gemm_tc": 2.0 * kl2 * N_v * d * min(V, chunk),
         "bwd_dh_gemm_tc": 2.0 * N_v * d * min(V, chunk), "bwd_dw_gemm_tc": 2.0 * N_v * d * min(V, chunk)}
     if dom in flops_per_launch:
         achieved = flops_per_launch[dom] / ((t_dom / n_dom) / 1e3) / 1e12
@@ -342,8 +356,9 @@ def run_gpu(args):
             gemm_tf[k] = round(flops_per_launch[k] / ((t / n) / 1e3) / 1e12, 1)
 
     out = {
-        "metric": "scored tokens/sec (fwd+bwd)" + (" [SFT distillation step]" if args.path == "sft"
-                                                    else ""),
+        "metric": "scored tokens/sec (fwd+bwd)" + {"sft": " [SFT distillation step]",
+                                                    "grpo-exact-kl": " [GRPO, exact KL]"}.get(
+                                                        args.path, ""),
         "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(step_ms, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
@@ -387,8 +402,9 @@ def main():
     ap.add_argument("--cpu-tokens", type=int, default=32)
     ap.add_argument("--ref-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--path", default="grpo", choices=["grpo", "sft"],
-                    help="grpo: the GRPO update (default); sft: the distillation loss step")
+    ap.add_argument("--path", default="grpo", choices=["grpo", "sft", "grpo-exact-kl"],
+                    help="grpo: the GRPO update (default); sft: the distillation loss step; "
+                         "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
     ap.add_argument("--cta-pair", type=int, default=0,
                     help="tensor-core tiles: 0 = single CTAs (default), 1 = CTA pairs (cta_group::2)")
     ap.add_argument("--scale", default="",

@@ -157,6 +157,30 @@ int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new
                  const int32_t* tools_used, const int32_t* tools_avail, int32_t n,
                  float lambda_tools, float* r_out, grpo_stream_t stream);
 
+/* Exact KL variant. Eq. 1 writes the full-distribution KL(pi_theta(.|c) || pi_ref(.|c)); with
+ * the frozen reference model of Alg. 1 (same d and V) its per-position term is
+ *   KL_t = sum_v p_tv (log p_tv - log q_tv),  p = softmax(W h_t),  q = softmax(W_ref h_ref_t).
+ * grpo_score_fwd_kl computes grpo_score_fwd's outputs plus lse_ref [S,T] and kl [S,T] (0 at
+ * unscored positions); both products stream through one tensor-core tile per 128 x 256 block,
+ * the logits of neither model reach memory. H_ref [S,T,d], W_ref [V,d] bf16. */
+int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
+                      int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
+                      int32_t T, int32_t d, int32_t V, float* logp, float* lse, float* entropy,
+                      int32_t* argmax, int32_t* valid_count, float* lse_ref, float* kl,
+                      void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
+/* grpo_loss_bwd with the exact KL: l_t = -surr_t + beta KL_t (the clipped surrogate as in
+ * grpo_loss_bwd), and dz_t = g_t (onehot(y_t) - p_t) + beta w_t p_t (log p_t - log q_t - KL_t)
+ * from both recomputed products; dH, dW as in grpo_loss_bwd (nothing flows to the frozen
+ * reference). logp, lse, lse_ref, kl are grpo_score_fwd_kl's outputs. bf16 only. */
+int grpo_loss_bwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
+                     int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
+                     int32_t T, int32_t d, int32_t V, const float* logp, const float* lse,
+                     const float* lse_ref, const float* kl, const float* old_logp,
+                     const float* adv, const int32_t* valid_count, float eps_low, float eps_high,
+                     float beta, int32_t agg, double norm, float* loss_out, void* dH, float* dW,
+                     void* workspace, size_t workspace_bytes, grpo_stream_t stream);
+
 /* Vocabulary-parallel (tensor-parallel) variant. The paper shards the policy over GPUs with
  * tensor parallelism (Sec. 6.3); sharding the LM head by vocabulary rows needs one exchange of
  * per-token statistics after the forward and one sum of dH after the backward.

@@ -85,7 +85,7 @@ struct Layout {
   long long rows_cap;
   int num_strips;
   int v_round;          // V rounded up to a multiple of 256
-  size_t seq_last, seq_tile_base, tiles, counts, zy, partials, g, seq_loss;
+  size_t seq_last, seq_tile_base, tiles, counts, zy, partials, partials2, g, cvec, seq_loss;
   size_t fixed_end;     // end of the regions that do not depend on the vocabulary chunk
 };
 
@@ -106,7 +106,10 @@ Layout make_layout(int S, int T, int d, int V, int dtype) {
   L.zy = off;             off = align256(off + sizeof(float) * P);
   L.partials = off;
   if (dtype == GRPO_BF16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  L.partials2 = off;      // exact-KL forward only
+  if (dtype == GRPO_BF16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
   L.g = off;              off = align256(off + sizeof(float) * P);
+  L.cvec = off;           off = align256(off + sizeof(float) * P);
   L.seq_loss = off;       off = align256(off + sizeof(float) * S);
   L.fixed_end = off;
   return L;
@@ -195,7 +198,9 @@ struct Views {
   int32_t* counts;
   float* zy;
   float4* partials;
+  float4* partials2;
   float* g;
+  float* cvec;
   float* seq_loss;
 };
 
@@ -209,7 +214,9 @@ Views views(void* ws, const Layout& L) {
   v.counts = reinterpret_cast<int32_t*>(b + L.counts);
   v.zy = reinterpret_cast<float*>(b + L.zy);
   v.partials = reinterpret_cast<float4*>(b + L.partials);
+  v.partials2 = reinterpret_cast<float4*>(b + L.partials2);
   v.g = reinterpret_cast<float*>(b + L.g);
+  v.cvec = reinterpret_cast<float*>(b + L.cvec);
   v.seq_loss = reinterpret_cast<float*>(b + L.seq_loss);
   return v;
 }
@@ -353,16 +360,24 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
                   const float* ref_logp, const float* adv, const int32_t* valid_count,
                   float eps_low, float eps_high, float beta, int32_t agg, double norm,
                   float* loss_out, void* dH, float* dW, void* workspace, size_t workspace_bytes,
-                  grpo_stream_t stream, int32_t v_offset = 0, bool dh_f32 = false) {
+                  grpo_stream_t stream, int32_t v_offset = 0, bool dh_f32 = false,
+                  const void* H_ref = nullptr, const void* W_ref = nullptr,
+                  const float* lse_ref = nullptr, const float* kl = nullptr) {
   if (!H || !W || !tokens || !mask || !logp || !lse || !valid_count || !loss_out || !dH || !dW)
     return GRPO_ERR_INVALID_ARG;
-  if (mode == 0 && (!old_logp || !adv)) return GRPO_ERR_INVALID_ARG;
+  if (mode != 1 && (!old_logp || !adv)) return GRPO_ERR_INVALID_ARG;
   if (mode == 0 && !ref_logp && beta != 0.f) return GRPO_ERR_INVALID_ARG;
-  if (mode != 0) {   // the distillation loss reads none of these
+  if (mode == 1) {   // the distillation loss reads none of these
     old_logp = logp;
     ref_logp = logp;
     adv = logp;
     beta = 0.f;
+  }
+  if (mode == 2) {   // exact KL: the reference model's hidden states and head replace ref_logp
+    if (!H_ref || !W_ref || !lse_ref || !kl) return GRPO_ERR_INVALID_ARG;
+    if (dtype != GRPO_BF16) return GRPO_ERR_UNSUPPORTED;
+    if (!aligned16(H_ref) || !aligned16(W_ref)) return GRPO_ERR_INVALID_ARG;
+    ref_logp = logp;
   }
   if (!shape_ok(S, T, d, V)) return GRPO_ERR_INVALID_ARG;
   GRPO_TRY(check_dtype_shape(dtype, d));
@@ -384,7 +399,8 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   }));
   GRPO_TRY(counted(GRPO_K_LOSS_TOKENS, st, [&] {
     return launch_loss_tokens(mask, logp, old_logp, ref, adv, valid_count, S, T, eps_low,
-                              eps_high, beta, agg, norm, mode, v.hdr, v.g, v.seq_loss, st);
+                              eps_high, beta, agg, norm, mode, v.hdr, v.g, v.seq_loss, st, kl,
+                              v.cvec);
   }));
   GRPO_TRY(counted(GRPO_K_LOSS_FINAL, st, [&] {
     return launch_loss_final(v.seq_loss, S, agg, norm, v.hdr, loss_out, st);
@@ -428,8 +444,11 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     dz = reinterpret_cast<__nv_bfloat16*>(wsb + L.fixed_end +
                                           align256(static_cast<size_t>(L.rows_cap) * d * 4));
   }
-  const bool pair = g_cta_pair.load() != 0;
-  CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn;
+  const bool pair = g_cta_pair.load() != 0 && mode != 2;   // exact-KL roles: single-CTA tiles
+  CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn, mapHrk, mapWrk;
+  if (mode == 2 && (!make_map(&mapHrk, H_ref, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+                    !make_map(&mapWrk, W_ref, d, V, d, kTileN)))
+    return GRPO_ERR_CUDA;
   const uint64_t P = static_cast<uint64_t>(S) * T;
   if (!make_map(&mapHk, H, d, P, d, kTileRows) ||
       !make_map(&mapWk, W, d, V, d, pair ? kTileN / 2 : kTileN) ||
@@ -443,6 +462,9 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   a.dh_f32 = dh_f32 ? 1 : 0;
   a.g = v.g;
   a.lse = lse;
+  a.c = v.cvec;
+  a.lse_ref = lse_ref;
+  a.kl = kl;
   a.dz = dz;
   a.dz_pitch = vc;
   a.dH = static_cast<__nv_bfloat16*>(dH);
@@ -454,6 +476,9 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     a.dh_mode = nchunks == 1 ? 0 : (c == 0 ? 1 : (c == nchunks - 1 ? 3 : 2));
     const long long vt = (a.vc_len + kTileN - 1) / kTileN;
     GRPO_TRY(counted(GRPO_K_BWD_DZ_GEMM, st, [&] {
+      if (mode == 2)
+        return launch_gemm(ROLE_DZ_KL, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, false), false,
+                           st, &mapHrk, &mapWrk);
       return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, pair), pair, st);
     }));
     GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
@@ -494,6 +519,61 @@ int grpo_sft_loss_bwd(const void* H, const void* W, int32_t dtype, const int32_t
   return loss_bwd_impl(1, H, W, dtype, tokens, mask, S, T, d, V, logp, lse, nullptr, nullptr,
                        nullptr, valid_count, 0.f, 0.f, 0.f, agg, norm, loss_out, dH, dW, workspace,
                        workspace_bytes, stream);
+}
+
+int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
+                      int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
+                      int32_t T, int32_t d, int32_t V, float* logp, float* lse, float* entropy,
+                      int32_t* argmax, int32_t* valid_count, float* lse_ref, float* kl,
+                      void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  if (!H || !W || !H_ref || !W_ref || !tokens || !mask || !logp || !lse || !entropy || !argmax ||
+      !valid_count || !lse_ref || !kl)
+    return GRPO_ERR_INVALID_ARG;
+  if (!shape_ok(S, T, d, V)) return GRPO_ERR_INVALID_ARG;
+  if (dtype != GRPO_BF16) return GRPO_ERR_UNSUPPORTED;
+  GRPO_TRY(check_dtype_shape(dtype, d));
+  if (!aligned16(H) || !aligned16(W) || !aligned16(H_ref) || !aligned16(W_ref))
+    return GRPO_ERR_INVALID_ARG;
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
+  const Layout L = make_layout(S, T, d, V, dtype);
+  if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const Views v = views(workspace, L);
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, valid_count, v.seq_last, st); }));
+  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
+    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
+  }));
+  const uint64_t P = static_cast<uint64_t>(S) * T;
+  CUtensorMap mapH, mapW, mapHr, mapWr;
+  if (!make_map(&mapH, H, d, P, d, kTileRows) || !make_map(&mapW, W, d, V, d, kTileN) ||
+      !make_map(&mapHr, H_ref, d, P, d, kTileRows) || !make_map(&mapWr, W_ref, d, V, d, kTileN))
+    return GRPO_ERR_CUDA;
+  GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
+  a.partials = v.partials;
+  a.partials2 = v.partials2;
+  a.zy = v.zy;
+  GRPO_TRY(counted(GRPO_K_FWD_GEMM, st, [&] {
+    return launch_gemm(ROLE_FWD_KL, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, false),
+                       false, st, &mapHr, &mapWr);
+  }));
+  return counted(GRPO_K_FWD_MERGE, st, [&] {
+    return launch_fwd_merge_kl(v.partials, v.partials2, L.rows_cap, L.num_strips, v.zy,
+                               v.seq_tile_base, tokens, mask, S, T, V, logp, lse, entropy, argmax,
+                               lse_ref, kl, v.hdr, st);
+  });
+}
+
+int grpo_loss_bwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
+                     int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
+                     int32_t T, int32_t d, int32_t V, const float* logp, const float* lse,
+                     const float* lse_ref, const float* kl, const float* old_logp,
+                     const float* adv, const int32_t* valid_count, float eps_low, float eps_high,
+                     float beta, int32_t agg, double norm, float* loss_out, void* dH, float* dW,
+                     void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
+  return loss_bwd_impl(2, H, W, dtype, tokens, mask, S, T, d, V, logp, lse, old_logp, logp, adv,
+                       valid_count, eps_low, eps_high, beta, agg, norm, loss_out, dH, dW,
+                       workspace, workspace_bytes, stream, 0, false, H_ref, W_ref, lse_ref, kl);
 }
 
 int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,

@@ -57,14 +57,14 @@ struct Dims {
 template <int ROLE>
 __device__ __forceinline__ Dims role_dims(const GemmArgs& a, int num_tiles) {
   Dims d;
-  if (ROLE == ROLE_FWD) {
+  if (ROLE == ROLE_FWD || ROLE == ROLE_FWD_KL) {
     d.num_m = num_tiles;
     d.num_n = a.num_strips;
-    d.num_kb = a.d / BK;
-  } else if (ROLE == ROLE_DZ) {
+    d.num_kb = (ROLE == ROLE_FWD_KL ? 2 : 1) * (a.d / BK);   // KL: policy, then reference
+  } else if (ROLE == ROLE_DZ || ROLE == ROLE_DZ_KL) {
     d.num_m = num_tiles;
     d.num_n = (a.vc_len + BN - 1) / BN;
-    d.num_kb = a.d / BK;
+    d.num_kb = (ROLE == ROLE_DZ_KL ? 2 : 1) * (a.d / BK);
   } else if (ROLE == ROLE_DH) {
     d.num_m = num_tiles;
     d.num_n = a.d / BN;
@@ -89,9 +89,16 @@ __device__ __forceinline__ void decode_unit(int u, int num_m, int num_n, int& m,
   n = within / gm;
 }
 
+// Roles whose tile holds two products (policy z in TMEM columns 0-255, reference z_ref in
+// 256-511): one accumulator buffer instead of two.
+template <int ROLE>
+struct Dual {
+  static constexpr bool value = (ROLE == ROLE_FWD_KL || ROLE == ROLE_DZ_KL);
+};
+
 template <int ROLE>
 __device__ __forceinline__ int acc_tiles_of_unit(const GemmArgs& a, int n) {
-  if (ROLE == ROLE_FWD) {
+  if (ROLE == ROLE_FWD || ROLE == ROLE_FWD_KL) {
     const int nvt = (a.V + BN - 1) / BN;
     return min(kFwdTilesPerStrip, nvt - n * kFwdTilesPerStrip);
   }
@@ -126,7 +133,8 @@ struct Sched {
 // producer: one thread per CTA
 // ------------------------------------------------------------------------------------------
 template <int ROLE, bool PAIR>
-__device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB, const GemmArgs& a,
+__device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
+                             const CUtensorMap* mapA2, const CUtensorMap* mapB2, const GemmArgs& a,
                              const Dims& dm, const Sched<PAIR>& sc, uint8_t* sA, uint8_t* sB,
                              uint64_t* full, uint64_t* empty, volatile int* abort_flag) {
   using C = Cfg<PAIR>;
@@ -144,7 +152,7 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB, c
     sc.m_of(mu, dm.num_m, m, m_load, m_ok);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     int hrow = 0;
-    if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
+    if (ROLE == ROLE_FWD || ROLE == ROLE_DZ || Dual<ROLE>::value) {
       const int2 tl = a.tiles[m_load];
       hrow = tl.x * a.T + tl.y;
     }
@@ -175,6 +183,14 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB, c
             const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
             load(dA, mapA, kb * BK, hrow);
             load(dB, mapB, kb * BK, vt * BN + b_col0);
+          } else if (Dual<ROLE>::value) {
+            // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
+            const int nk = dm.num_kb / 2;
+            const bool second = kb >= nk;
+            const int kk = second ? kb - nk : kb;
+            const int vt = (ROLE == ROLE_FWD_KL) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
+            load(dA, second ? mapA2 : mapA, kk * BK, hrow);
+            load(dB, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
           } else if (ROLE == ROLE_DH) {
             load(dA, mapA, kb * BK, m_load * BM);
 #pragma unroll
@@ -241,6 +257,7 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
       }
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + buf * BN;
+      const int nk = Dual<ROLE>::value ? dm.num_kb / 2 : dm.num_kb;
       for (int kb = 0; kb < dm.num_kb; ++kb) {
         if (!mbar_wait_bounded(&full[stage], phase, abort_flag, a.hdr,
                                WHERE_GEMM_BASE + ROLE * 16 + 3)) {
@@ -250,6 +267,10 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
         tc_fence_after();
         const uint32_t a0 = smem_u32(sA + stage * C::A_STAGE);
         const uint32_t b0 = smem_u32(sB + stage * C::B_STAGE);
+        // dual roles: the reference product goes to the other TMEM half, accumulating afresh
+        const bool second = Dual<ROLE>::value && kb >= nk;
+        const uint32_t dst = second ? d_tmem + BN : d_tmem;
+        const int kr = second ? kb - nk : kb;
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k) {
           const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, BOX_MN, 1024)
@@ -257,9 +278,9 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
           const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, BOX_MN, 1024)
                                    : sdesc_sw128(b0 + k * 32, 16, 1024);
           if (PAIR) {
-            umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            umma_bf16_pair(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
           } else {
-            umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            umma_bf16(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
           }
         }
         // frees the smem stage (in both CTAs of a pair) once these MMAs have read it
@@ -279,8 +300,12 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
       } else {
         umma_commit(&accf[buf]);
       }
-      buf ^= 1u;
-      if (buf == 0) bphase ^= 1u;
+      if (Dual<ROLE>::value) {         // one buffer spanning all of TMEM
+        bphase ^= 1u;
+      } else {
+        buf ^= 1u;
+        if (buf == 0) bphase ^= 1u;
+      }
     }
   }
   // Make sure no MMA is still writing tensor memory when it is released.
@@ -412,6 +437,144 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
             make_float4(rm, rs, ru, __int_as_float(ri));
       if (found) a.zy[pos] = zyv;
 
+    } else if (ROLE == ROLE_FWD_KL) {
+      // policy z in columns 0-255, reference z_ref in 256-511 of the one buffer
+      const int2 tl = a.tiles[m_load];
+      const bool rv = m_ok && tl.y + r < a.T;
+      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] : -1;
+      float rm = -INFINITY, rs = 0.f, ru = 0.f, rc = 0.f, zyv = 0.f;
+      float qm = -INFINITY, qs = 0.f;
+      int ri = 0;
+      bool found = false;
+      const int nacc = acc_tiles_of_unit<ROLE>(a, n);
+      for (int t = 0; t < nacc; ++t) {
+        if (!epi_wait(&accf[0], bphase, abort_flag, a.hdr, where)) return;
+        tc_fence_after();
+        const int vbase = (n * kFwdTilesPerStrip + t) * BN;
+        for (int c = 0; c < BN / 32; ++c) {
+          const int v0 = vbase + c * 32;
+          if (v0 >= a.V) break;
+          float x[32], xr[32];
+          tmem_load_32cols(t_row + c * 32, x);
+          tmem_load_32cols(t_row + BN + c * 32, xr);
+          const int nvalid = a.V - v0;
+          if (nvalid < 32) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j >= nvalid) {
+                x[j] = -1.0e30f;
+                xr[j] = -1.0e30f;
+              }
+          }
+          float cm = x[0], cq = xr[0];
+          int ci = 0;
+#pragma unroll
+          for (int j = 1; j < 32; ++j) {
+            if (x[j] > cm) {
+              cm = x[j];
+              ci = j;
+            }
+            cq = fmaxf(cq, xr[j]);
+          }
+          if (cm > rm) {
+            const float scl = ex2_approx((rm - cm) * kLog2e);
+            rs *= scl;
+            ru *= scl;
+            rc *= scl;
+            rm = cm;
+            ri = v0 + ci;
+          }
+          if (cq > qm) {
+            qs *= ex2_approx((qm - cq) * kLog2e);
+            qm = cq;
+          }
+          const float ml = rm * kLog2e, ql = qm * kLog2e;
+          float ps = 0.f, pu = 0.f, pc = 0.f, qq = 0.f;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float e = ex2_approx(fmaf(x[j], kLog2e, -ml));
+            ps += e;
+            pu = fmaf(e, x[j], pu);
+            pc = fmaf(e, xr[j], pc);
+            qq += ex2_approx(fmaf(xr[j], kLog2e, -ql));
+          }
+          rs += ps;
+          ru += pu;
+          rc += pc;
+          qs += qq;
+          const int rel = y - v0;
+          if (rel >= 0 && rel < 32) {
+            float zt = x[0];
+#pragma unroll
+            for (int j = 1; j < 32; ++j)
+              if (j == rel) zt = x[j];
+            zyv = zt;
+            found = true;
+          }
+        }
+        epi_release<PAIR>(&acce[0], lane, sc.rank);
+        bphase ^= 1u;
+      }
+      if (m_ok) {
+        const long long at = static_cast<long long>(n) * a.rows_cap +
+                             static_cast<long long>(m) * BM + r;
+        a.partials[at] = make_float4(rm, rs, ru, __int_as_float(ri));
+        a.partials2[at] = make_float4(rc, qm, qs, 0.f);
+      }
+      if (found) a.zy[pos] = zyv;
+
+    } else if (ROLE == ROLE_DZ_KL) {
+      // dz = g (onehot - p) + c p (log p - log q - KL), p from z, q from z_ref
+      const int2 tl = a.tiles[m_load];
+      const bool rv = m_ok && tl.y + r < a.T;
+      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const bool act = rv && a.mask[pos] != 0;
+      const float gt = act ? a.g[pos] : 0.f;
+      const float ct = act ? a.c[pos] : 0.f;
+      const float lse = act ? a.lse[pos] : 0.f;
+      const float lser = act ? a.lse_ref[pos] : 0.f;
+      const float klt = act ? a.kl[pos] : 0.f;
+      const int y = act ? a.tokens[pos] : -1;
+      if (!epi_wait(&accf[0], bphase, abort_flag, a.hdr, where)) return;
+      tc_fence_after();
+      __nv_bfloat16* dst_row =
+          a.dz + (static_cast<size_t>(m_load) * BM + r) * static_cast<size_t>(a.dz_pitch);
+      for (int c = 0; c < BN / 32; ++c) {
+        const int vloc = n * BN + c * 32;
+        const int v0 = a.vc0 + vloc;
+        float x[32], xr[32];
+        tmem_load_32cols(t_row + c * 32, x);
+        tmem_load_32cols(t_row + BN + c * 32, xr);
+        if (!m_ok) continue;
+        uint32_t pk[16];
+        if (act) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            float dv[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int v = v0 + 2 * j + e;
+              const float lp = x[2 * j + e] - lse;              // log p
+              const float p = ex2_approx(lp * kLog2e);
+              const float lq = xr[2 * j + e] - lser;            // log q
+              const float val = gt * ((v == y ? 1.f : 0.f) - p) + ct * p * (lp - lq - klt);
+              dv[e] = v < a.V ? val : 0.f;
+            }
+            pk[j] = pack_bf16x2(dv[0], dv[1]);
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) pk[j] = 0u;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(dst_row + vloc);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+      }
+      epi_release<PAIR>(&acce[0], lane, sc.rank);
+      bphase ^= 1u;
+
     } else if (ROLE == ROLE_DZ) {
       const int2 tl = a.tiles[m_load];
       const bool rv = m_ok && tl.y + r < a.T;
@@ -533,6 +696,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
 // ------------------------------------------------------------------------------------------
 template <int ROLE, bool PAIR>
 __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtensorMap* mapB,
+                                          const CUtensorMap* mapA2, const CUtensorMap* mapB2,
                                           const GemmArgs& args) {
   using C = Cfg<PAIR>;
   extern __shared__ uint8_t smem_raw[];
@@ -567,6 +731,10 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(mapA);
     tma_prefetch_desc(mapB);
+    if (Dual<ROLE>::value) {
+      tma_prefetch_desc(mapA2);
+      tma_prefetch_desc(mapB2);
+    }
   }
   if (warp == 1) {
     if (PAIR) {
@@ -590,7 +758,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
 
   if (warp == 0) {
     if (lane == 0)
-      run_producer<ROLE, PAIR>(mapA, mapB, args, dm, sc, sA, sB, full, empty, abort_flag);
+      run_producer<ROLE, PAIR>(mapA, mapB, mapA2, mapB2, args, dm, sc, sA, sB, full, empty,
+                               abort_flag);
   } else if (warp == 1) {
     if (lane == 0)
       run_mma<ROLE, PAIR>(args, dm, sc, sA, sB, full, empty, accf, acce, drain, tmem_base,
@@ -618,21 +787,23 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
 template <int ROLE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+            const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
             const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, false>(&mapA, &mapB, args);
+  gemm_body<ROLE, false>(&mapA, &mapB, &mapA2, &mapB2, args);
 }
 
 template <int ROLE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_pair(const __grid_constant__ CUtensorMap mapA,
                  const __grid_constant__ CUtensorMap mapB, const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, true>(&mapA, &mapB, args);
+  gemm_body<ROLE, true>(&mapA, &mapB, &mapA, &mapB, args);
 }
 
 template <int ROLE>
 cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const GemmArgs& args,
-                        int grid, bool pair, cudaStream_t st) {
-  if (pair) {
+                        int grid, bool pair, cudaStream_t st, const CUtensorMap& mapA2,
+                        const CUtensorMap& mapB2) {
+  if (pair && !Dual<ROLE>::value) {
     const size_t smem = Cfg<true>::SMEM;
     cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair<ROLE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -644,7 +815,7 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
     cudaError_t e = cudaFuncSetAttribute(tc_gemm<ROLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    tc_gemm<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+    tc_gemm<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, mapA2, mapB2, args);
   }
   return cudaGetLastError();
 }
@@ -654,12 +825,21 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
 size_t gemm_smem_bytes() { return SMEM_BYTES; }
 
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, bool pair, cudaStream_t st) {
+                        const GemmArgs& args, int grid, bool pair, cudaStream_t st,
+                        const CUtensorMap* mapA2, const CUtensorMap* mapB2) {
+  const CUtensorMap& a2 = mapA2 ? *mapA2 : mapA;
+  const CUtensorMap& b2 = mapB2 ? *mapB2 : mapB;
   switch (role) {
-    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, pair, st);
-    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, pair, st);
-    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, pair, st);
-    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, pair, st);
+    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, pair, st, a2, b2);
+    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, pair, st, a2, b2);
+    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, pair, st, a2, b2);
+    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, pair, st, a2, b2);
+    case ROLE_FWD_KL:
+      if (!mapA2 || !mapB2 || pair) return cudaErrorInvalidValue;
+      return launch_role<ROLE_FWD_KL>(mapA, mapB, args, grid, false, st, a2, b2);
+    case ROLE_DZ_KL:
+      if (!mapA2 || !mapB2 || pair) return cudaErrorInvalidValue;
+      return launch_role<ROLE_DZ_KL>(mapA, mapB, args, grid, false, st, a2, b2);
     default: return cudaErrorInvalidValue;
   }
 }

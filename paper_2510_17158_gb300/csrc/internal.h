@@ -20,7 +20,11 @@ constexpr int kTileN = 256;
 // Vocabulary tiles merged on chip by one forward work unit before it writes partial statistics.
 constexpr int kFwdTilesPerStrip = 8;
 
-enum GemmRole : int { ROLE_FWD = 0, ROLE_DZ = 1, ROLE_DH = 2, ROLE_DW = 3 };
+// FWD_KL / DZ_KL: the forward / dz roles with a second product z_ref = W_ref h_ref (the frozen
+// reference model) in the other half of tensor memory, for Eq. 1's exact KL term.
+enum GemmRole : int {
+  ROLE_FWD = 0, ROLE_DZ = 1, ROLE_DH = 2, ROLE_DW = 3, ROLE_FWD_KL = 4, ROLE_DZ_KL = 5
+};
 
 // Arguments of the tcgen05 GEMM kernels (one struct for the four roles).
 struct GemmArgs {
@@ -53,6 +57,12 @@ struct GemmArgs {
   int v_offset;
   // DH: write the final dH in f32 (a shard's partial sum) instead of H's dtype
   int dh_f32;
+  // FWD_KL: second set of per-(strip, row) statistics (sum e^{z-m} z_ref, m_ref, s_ref, 0)
+  float4* partials2;
+  // DZ_KL: per-position log-normaliser of the reference, exact KL, and its coefficient beta*w
+  const float* lse_ref;
+  const float* kl;
+  const float* c;
 };
 
 // Launches (all asynchronous on `st`; return the cudaError_t of the launch).
@@ -68,11 +78,20 @@ cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num
                              const int32_t* tokens, const uint8_t* mask, int S, int T, int V,
                              float* logp, float* lse, float* entropy, int32_t* argmax,
                              WsHeader* hdr, cudaStream_t st);
+// mode 0 GRPO (per-token KL estimator), 1 SFT, 2 GRPO with the exact KL (reads kl, writes
+// c = beta * w per position).
 cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const float* old_logp,
                                const float* ref_logp, const float* adv,
                                const int32_t* valid_count, int S, int T, float eps_low,
                                float eps_high, float beta, int agg, double norm, int mode,
-                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st);
+                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st,
+                               const float* kl = nullptr, float* c = nullptr);
+cudaError_t launch_fwd_merge_kl(const float4* partials, const float4* partials2,
+                                long long rows_cap, int num_strips, const float* zy,
+                                const int32_t* seq_tile_base, const int32_t* tokens,
+                                const uint8_t* mask, int S, int T, int V, float* logp, float* lse,
+                                float* entropy, int32_t* argmax, float* lse_ref, float* kl,
+                                WsHeader* hdr, cudaStream_t st);
 cudaError_t launch_rewards(const uint8_t* correct, const float* t_base, const float* t_new,
                            const int32_t* used, const int32_t* avail, int n, float lambda_tools,
                            float* r, cudaStream_t st);
@@ -106,7 +125,9 @@ bool gemm_pair_mode();
 // tcgen05 GEMM launches. `grid` = persistent CTAs.
 size_t gemm_smem_bytes();
 // pair = true: CTA-pair kernels (clusters of 2, cta_group::2); `grid` must then be even.
+// mapA2 / mapB2 (H_ref, W_ref) are read by the KL roles only (single-CTA tiles).
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, bool pair, cudaStream_t st);
+                        const GemmArgs& args, int grid, bool pair, cudaStream_t st,
+                        const CUtensorMap* mapA2 = nullptr, const CUtensorMap* mapB2 = nullptr);
 
 }  // namespace grpo

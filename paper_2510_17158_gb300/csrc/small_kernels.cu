@@ -215,6 +215,71 @@ __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_
   argmax[pos] = idx;
 }
 
+// Merge for the exact-KL forward: also combines sum e^{z-m} z_ref and the reference model's
+// (m_ref, s_ref) into lse_ref and KL_t = E_p[z] - lse - E_p[z_ref] + lse_ref.
+__global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
+                               const float4* __restrict__ partials2, long long rows_cap,
+                               int num_strips, const float* __restrict__ zy,
+                               const int32_t* __restrict__ seq_tile_base,
+                               const int32_t* __restrict__ tokens,
+                               const uint8_t* __restrict__ mask, int S, int T, int V,
+                               float* __restrict__ logp, float* __restrict__ lse_out,
+                               float* __restrict__ entropy, int32_t* __restrict__ argmax,
+                               float* __restrict__ lse_ref, float* __restrict__ kl,
+                               WsHeader* hdr) {
+  const long long pos = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (pos >= static_cast<long long>(S) * T) return;
+  if (mask[pos] == 0) {
+    logp[pos] = 0.f;
+    lse_out[pos] = 0.f;
+    entropy[pos] = 0.f;
+    argmax[pos] = -1;
+    lse_ref[pos] = 0.f;
+    kl[pos] = 0.f;
+    return;
+  }
+  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
+  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
+                        (t % kTileRows);
+  float M = -INFINITY, Mr = -INFINITY;
+  int idx = 0;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    const float4 q = partials2[static_cast<long long>(j) * rows_cap + row];
+    if (p.x > M) {
+      M = p.x;
+      idx = __float_as_int(p.w);
+    }
+    Mr = fmaxf(Mr, q.y);
+  }
+  float Ssum = 0.f, U = 0.f, C = 0.f, Sr = 0.f;
+  for (int j = 0; j < num_strips; ++j) {
+    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
+    const float4 q = partials2[static_cast<long long>(j) * rows_cap + row];
+    const float sc = ex2_approx((p.x - M) * kLog2e);
+    Ssum = fmaf(p.y, sc, Ssum);
+    U = fmaf(p.z, sc, U);
+    C = fmaf(q.x, sc, C);
+    Sr = fmaf(q.z, ex2_approx((q.y - Mr) * kLog2e), Sr);
+  }
+  const float lse = M + logf(Ssum);
+  const float lser = Mr + logf(Sr);
+  const int y = tokens[pos];
+  float lp;
+  if (y < 0 || y >= V) {
+    record_error(hdr, ST_TOKEN_RANGE, WHERE_MERGE_TOKEN);
+    lp = __int_as_float(0x7fc00000);
+  } else {
+    lp = zy[pos] - lse;
+  }
+  logp[pos] = lp;
+  lse_out[pos] = lse;
+  entropy[pos] = lse - U / Ssum;
+  argmax[pos] = idx;
+  lse_ref[pos] = lser;
+  kl[pos] = fmaxf(0.f, (U - C) / Ssum - lse + lser);   // >= 0; rounding can dip below 0
+}
+
 // ------------------------------------------------------------------------------------------
 // Per-token loss terms and g_t = dL/dlogp_t; one block per sequence, fixed-order block sum.
 // ------------------------------------------------------------------------------------------
@@ -241,10 +306,11 @@ __global__ void __launch_bounds__(kLossThreads)
                   const float* __restrict__ adv, const int32_t* __restrict__ valid_count, int S,
                   int T, float eps_low, float eps_high, float beta, int agg, double norm,
                   int mode, const WsHeader* hdr, float* __restrict__ g,
-                  float* __restrict__ seq_loss) {
+                  float* __restrict__ seq_loss, const float* __restrict__ kl,
+                  float* __restrict__ cvec) {
   __shared__ float sh[32];
   const int i = blockIdx.x;
-  const float A = mode == 0 ? adv[i] : 0.f;
+  const float A = mode != 1 ? adv[i] : 0.f;
   const int n_i = valid_count[i];
   float w;
   if (agg == 0) {
@@ -273,7 +339,11 @@ __global__ void __launch_bounds__(kLossThreads)
       float dell = 0.f;
       const bool active = (A >= 0.f) ? (rho <= hi) : (rho >= lo);
       if (active) dell = -A * rho;
-      if (beta != 0.f) {
+      if (mode == 2) {
+        // exact KL (Eq. 1): its gradient enters dz directly with coefficient beta * w
+        ell = fmaf(beta, kl[pos], ell);
+        cvec[pos] = beta * w;
+      } else if (beta != 0.f) {
         const float delta = ref_logp[pos] - lp;
         const float ed = expf(delta);
         ell = fmaf(beta, ed - delta - 1.f, ell);
@@ -281,6 +351,8 @@ __global__ void __launch_bounds__(kLossThreads)
       }
       acc += ell;
       gt = w * dell;
+    } else if (mode == 2) {
+      cvec[pos] = 0.f;
     }
     g[pos] = gt;
   }
@@ -655,10 +727,24 @@ cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const flo
                                const float* ref_logp, const float* adv,
                                const int32_t* valid_count, int S, int T, float eps_low,
                                float eps_high, float beta, int agg, double norm, int mode,
-                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st) {
+                               const WsHeader* hdr, float* g, float* seq_loss, cudaStream_t st,
+                               const float* kl, float* c) {
   k_loss_tokens<<<S, kLossThreads, 0, st>>>(mask, logp, old_logp, ref_logp, adv, valid_count, S,
                                             T, eps_low, eps_high, beta, agg, norm, mode, hdr, g,
-                                            seq_loss);
+                                            seq_loss, kl, c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_merge_kl(const float4* partials, const float4* partials2,
+                                long long rows_cap, int num_strips, const float* zy,
+                                const int32_t* seq_tile_base, const int32_t* tokens,
+                                const uint8_t* mask, int S, int T, int V, float* logp, float* lse,
+                                float* entropy, int32_t* argmax, float* lse_ref, float* kl,
+                                WsHeader* hdr, cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  k_fwd_merge_kl<<<static_cast<unsigned>((P + 255) / 256), 256, 0, st>>>(
+      partials, partials2, rows_cap, num_strips, zy, seq_tile_base, tokens, mask, S, T, V, logp,
+      lse, entropy, argmax, lse_ref, kl, hdr);
   return cudaGetLastError();
 }
 

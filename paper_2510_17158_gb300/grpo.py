@@ -64,6 +64,11 @@ def _declare(lib):
         "grpo_sft_loss_bwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                              _p, _p, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
         "grpo_rewards": (ctypes.c_int, [_p, _p, _p, _p, _p, _i32, _f32, _p, _p]),
+        "grpo_score_fwd_kl": (ctypes.c_int, [_p, _p, _p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32,
+                                             _p, _p, _p, _p, _p, _p, _p, _p, _sz, _p]),
+        "grpo_loss_bwd_kl": (ctypes.c_int, [_p, _p, _p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32,
+                                            _p, _p, _p, _p, _p, _p, _p, _f32, _f32, _f32, _i32,
+                                            _f64, _p, _p, _p, _p, _sz, _p]),
         "grpo_score_fwd_shard": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32,
                                                 _i32, _i32, _p, _p, _p, _sz, _p]),
         "grpo_merge_shard_stats": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _p, _p,
@@ -319,6 +324,52 @@ def grpo_rewards(correct, t_base, t_new, tools_used, tools_avail, lambda_tools=0
                              _stream(stream))
     _check(st, "grpo_rewards")
     return r_out
+
+
+def grpo_score_fwd_kl(H, W, H_ref, W_ref, tokens, mask, ws: Workspace, out: Optional[dict] = None,
+                      stream=None) -> dict:
+    """Forward with the exact per-token KL to the reference model: grpo_score_fwd's outputs plus
+    lse_ref and kl."""
+    S, T, d = H.shape
+    V = W.shape[0]
+    for name, t, shape in (("H", H, (S, T, d)), ("W", W, (V, d)), ("H_ref", H_ref, (S, T, d)),
+                           ("W_ref", W_ref, (V, d))):
+        _need(t, name, torch.bfloat16, shape)
+    _need(tokens, "tokens", torch.int32, (S, T))
+    _need(mask, "mask", torch.uint8, (S, T))
+    if out is None:
+        f = dict(dtype=torch.float32, device=H.device)
+        out = {k: torch.empty((S, T), **f) for k in ("logp", "lse", "entropy", "lse_ref", "kl")}
+        out["argmax"] = torch.empty((S, T), dtype=torch.int32, device=H.device)
+        out["valid_count"] = torch.empty((S,), dtype=torch.int32, device=H.device)
+    st = _lib().grpo_score_fwd_kl(_ptr(H), _ptr(W), _ptr(H_ref), _ptr(W_ref), GRPO_BF16,
+                                  _ptr(tokens), _ptr(mask), S, T, d, V, _ptr(out["logp"]),
+                                  _ptr(out["lse"]), _ptr(out["entropy"]), _ptr(out["argmax"]),
+                                  _ptr(out["valid_count"]), _ptr(out["lse_ref"]), _ptr(out["kl"]),
+                                  ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "grpo_score_fwd_kl")
+    return out
+
+
+def grpo_loss_bwd_kl(H, W, H_ref, W_ref, tokens, mask, fwd: dict, old_logp, adv,
+                     ws: Workspace, eps_low=0.2, eps_high=0.2, beta=0.04, agg="seq_mean",
+                     norm=0.0, out: Optional[dict] = None, stream=None) -> dict:
+    """GRPO loss with the exact KL and its gradients; `fwd` is grpo_score_fwd_kl's output."""
+    S, T, d = H.shape
+    V = W.shape[0]
+    if out is None:
+        out = {"loss": torch.empty((1,), dtype=torch.float32, device=H.device),
+               "dH": torch.empty_like(H),
+               "dW": torch.empty((V, d), dtype=torch.float32, device=H.device)}
+    st = _lib().grpo_loss_bwd_kl(_ptr(H), _ptr(W), _ptr(H_ref), _ptr(W_ref), GRPO_BF16,
+                                 _ptr(tokens), _ptr(mask), S, T, d, V, _ptr(fwd["logp"]),
+                                 _ptr(fwd["lse"]), _ptr(fwd["lse_ref"]), _ptr(fwd["kl"]),
+                                 _ptr(old_logp), _ptr(adv), _ptr(fwd["valid_count"]),
+                                 float(eps_low), float(eps_high), float(beta), AGG_MODES[agg],
+                                 float(norm), _ptr(out["loss"]), _ptr(out["dH"]), _ptr(out["dW"]),
+                                 ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "grpo_loss_bwd_kl")
+    return out
 
 
 def grpo_score_fwd_shard(H, W_shard, tokens, mask, v_offset: int, V_total: int, ws: Workspace,

@@ -248,6 +248,29 @@ def make_batch_torch(w: Workload, device: str = "cuda", sample_chunk_tokens: int
                  torch.from_numpy(offsets).to(device), noise_old.float(), noise_ref.float())
 
 
+def reference_model_inputs(batch: Batch, seed: int = 7, h_sigma: float = 0.3,
+                           w_sigma: float = 0.004):
+    """Hidden states and LM head of the frozen reference model (Alg. 1) for a batch: the policy's
+    tensors plus Gaussian perturbations (h: sigma h_sigma, then rescaled to the policy token's
+    RMS; W: sigma w_sigma), in the batch's dtype and on its device (seeded torch generator on
+    that device). Draws only."""
+    dev = batch.H.device
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed)
+    Hr = torch.empty_like(batch.H)
+    for i in range(batch.H.shape[0]):           # one sequence at a time bounds the f32 scratch
+        h = batch.H[i].float()
+        x = h + h_sigma * torch.randn(h.shape, generator=gen, device=dev)
+        x = x * torch.sqrt(torch.mean(h * h, dim=-1, keepdim=True) /
+                           torch.mean(x * x, dim=-1, keepdim=True))
+        Hr[i].copy_(x)
+    Wr = torch.empty_like(batch.W)
+    for v0 in range(0, batch.W.shape[0], 16384):
+        wv = batch.W[v0:v0 + 16384].float()
+        Wr[v0:v0 + 16384].copy_(wv + w_sigma * torch.randn(wv.shape, generator=gen, device=dev))
+    return Hr, Wr
+
+
 def token_count_mean(w: Workload) -> float:
     """Expected number of scored tokens of a workload (mean of its length law, no holes)."""
     return w.S * min(w.T, (w.len_lo + w.len_hi) / 2.0)
@@ -259,4 +282,4 @@ def lm_head_flops(n_tokens: int, d: int, V: int) -> float:
 
 
 __all__ = ["Workload", "WORKLOADS", "Batch", "make_batch_numpy", "make_batch_torch",
-           "token_count_mean", "lm_head_flops"]
+           "reference_model_inputs", "token_count_mean", "lm_head_flops"]

@@ -78,3 +78,40 @@ def test_rewards_feed_group_advantages():
     adv_o = oracle.group_advantages(r.cpu().numpy(), go)
     np.testing.assert_allclose(r.cpu().numpy(), r_o, rtol=2e-6, atol=2e-6)
     np.testing.assert_allclose(adv, adv_o, rtol=1e-5, atol=2e-6)
+
+
+@pytest.mark.parametrize("name,over", [
+    ("g8_t1k_d2048_v32k", dict(prompts=1, group_sizes=(4,), T=260, len_lo=60, len_hi=260)),
+    ("g16_t16k_d5120_v152k", dict(group_sizes=(3,), prompts=1, T=140, len_lo=30, len_hi=140)),
+])
+def test_exact_kl_parity(name, over):
+    """Eq. 1's KL taken exactly over the vocabulary against a frozen reference model."""
+    from paper_2510_17158_gb300.synthetic import reference_model_inputs
+    from tests.parity_util import oracle_inputs
+    b = make_batch_numpy(WORKLOADS[name].scaled(**over))
+    w = b.workload
+    Hr, Wr = reference_model_inputs(b)
+    H, W, tok, mask = (t.cuda() for t in (b.H, b.W, b.tokens, b.mask))
+    S, T, d = H.shape
+    ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
+    old, _ = oracle_inputs(b, old_scale=2.0)
+    adv = G.group_advantages(b.rewards.cuda(), b.group_offsets.cuda(), ws)
+    f = G.grpo_score_fwd_kl(H, W, Hr.cuda(), Wr.cuda(), tok, mask, ws)
+    r = G.grpo_loss_bwd_kl(H, W, Hr.cuda(), Wr.cuda(), tok, mask, f, torch.from_numpy(old).cuda(),
+                           adv, ws, eps_low=w.eps, eps_high=w.eps, beta=0.5)
+    torch.cuda.synchronize()
+    assert G.grpo_last_device_error(ws)[0] == 0
+    o = oracle.grpo_step_exact_kl(b.H.double().numpy(), b.W.double().numpy(),
+                                  Hr.double().numpy(), Wr.double().numpy(), b.tokens.numpy(),
+                                  b.mask.numpy(), b.rewards.numpy(), b.group_offsets.numpy(),
+                                  old.astype(np.float64), w.eps, w.eps, 0.5)
+    m = b.mask.numpy() != 0
+    for k in ("logp", "lse", "entropy", "lse_ref", "kl"):
+        e = np.abs(f[k].cpu().numpy()[m] - o[k][m]).max()
+        assert e <= LOGP_ATOL, (k, e)
+    loss = float(r["loss"].item())
+    assert abs(loss - o["loss"]) <= 1e-3 * max(abs(o["loss"]), o["loss_abs_mass"]), (loss, o["loss"])
+    e_h = rel_fro(r["dH"].float().cpu().numpy(), o["dH"])
+    e_w = rel_fro(r["dW"].cpu().numpy(), o["dW"])
+    assert e_h <= GRAD_RTOL and e_w <= GRAD_RTOL, (e_h, e_w)
+    print(name, "kl mean", float(o["kl"][m].mean()), "loss", loss, o["loss"], "dH", e_h, "dW", e_w)
