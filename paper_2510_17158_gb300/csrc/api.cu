@@ -152,6 +152,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
+#ifndef GRPO_TMA_L2_PROMOTION
+#define GRPO_TMA_L2_PROMOTION CU_TENSOR_MAP_L2_PROMOTION_L2_256B
+#endif
+
 // 2-D bf16 tensor [outer, inner] (inner contiguous, row pitch `pitch_elems`), box
 // [box_outer, 64], 128-byte swizzle, out-of-range elements read as zero.
 bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
@@ -164,7 +168,7 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer
   cuuint32_t es[2] = {1, 1};
   const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
                         strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_SWIZZLE_128B, GRPO_TMA_L2_PROMOTION,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }

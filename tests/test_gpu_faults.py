@@ -70,3 +70,30 @@ def test_bad_group_offsets_set_status():
     a = G.group_advantages(r, go, ws)
     assert G.grpo_last_device_error(ws)[0] == 0
     assert np.isfinite(a.cpu().numpy()).all()
+
+
+def test_stalled_pipeline_times_out_in_cta_pair_mode():
+    """The same injected stall with CTA-pair tiles: the leader's MMA wait runs out, both CTAs of
+    every pair leave through their bounded waits and the final cluster barrier, and the next
+    call is correct."""
+    b, (H, W, tok, mask) = _small()
+    S, T, d = H.shape
+    ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
+    G.grpo_set_cta_pair(True)
+    try:
+        good = {k: v.clone() for k, v in G.grpo_score_fwd(H, W, tok, mask, ws).items()}
+        assert G.grpo_last_device_error(ws)[0] == 0
+        G.grpo_debug_inject_stall(True)
+        try:
+            G.grpo_score_fwd(H, W, tok, mask, ws)
+            st, where = G.grpo_last_device_error(ws)
+        finally:
+            G.grpo_debug_inject_stall(False)
+        assert st == TIMEOUT, (st, where)
+        again = G.grpo_score_fwd(H, W, tok, mask, ws)
+        torch.cuda.synchronize()
+        assert G.grpo_last_device_error(ws)[0] == 0
+        for k in ("logp", "lse", "entropy", "argmax"):
+            assert torch.equal(again[k], good[k]), k
+    finally:
+        G.grpo_set_cta_pair(False)

@@ -130,3 +130,18 @@ def test_pair_tiles_match_oracle_and_single_cta_tiles():
     print(compare(b, g1, o), compare(b, g2, o))
     for k in ("logp", "lse", "entropy"):
         assert float((g1[k] - g2[k]).abs().max()) <= 1e-4
+
+
+def test_chunked_backward_full_vocabulary_partial_last_chunk():
+    """V = 151936 in vocabulary chunks of 40960 (the last one 29056 wide, not a multiple of
+    256): the f32 dH accumulator path across four chunks meets the parity bar."""
+    from paper_2510_17158_gb300 import grpo as G
+    b = _batch("d4096_v152k")
+    old, ref = oracle_inputs(b)
+    S, T, d = b.H.shape
+    need = G.grpo_workspace_bytes(S, T, d, b.W.shape[0], b.H.dtype, 40960)
+    full = G.grpo_workspace_bytes(S, T, d, b.W.shape[0], b.H.dtype, 0)
+    assert need < full
+    g = run_gpu(b, old, ref, 0.2, 0.2, 0.04, vocab_chunk=40960)
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
+    print(compare(b, g, o))
