@@ -100,8 +100,8 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
  * Arguments, outputs and results are those of grpo_score_fwd, except:
  *  - the scratch is a GRPO_STATIC_SCRATCH_BYTES (64 MiB) __device__ array inside the library,
  *    held on every GPU that loads the library until the process exits. A batch whose scratch
- *    (about 16 * S*ceil(T/128)*128 * ceil(V/2048) + 4*S*T bytes for bf16) does not fit returns
- *    GRPO_ERR_WORKSPACE before anything is enqueued;
+ *    (for bf16 about R * (16 * ceil(V/2048) + 2 * d + 4) + 8 * S*T bytes, R = S*T rounded up to
+ *    a multiple of 128) does not fit returns GRPO_ERR_WORKSPACE before anything is enqueued;
  *  - it allocates nothing and calls no allocating routine;
  *  - the first call made with a given device current looks up the array's device address
  *    (cudaGetSymbolAddress) and caches it: make that first call before any stream capture;
@@ -201,8 +201,8 @@ int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
 /* Merges the statistics of all shards after they were exchanged (e.g. all-gathered so that
  * stats is [num_shards, S, T, 4] and zy [num_shards, S, T]) into grpo_score_fwd's outputs:
  * lse = M + log sum_p s_p e^{m_p - M}, logp = z_y - lse, entropy = lse - U/S, argmax = lowest
- * global index attaining M; valid_count as in grpo_score_fwd. Needs 256 + 4*S bytes of
- * workspace (rounded up to 256). */
+ * global index attaining M; valid_count as in grpo_score_fwd. Needs 256 bytes of
+ * workspace. */
 int grpo_merge_shard_stats(const float* stats, const float* zy, int32_t num_shards,
                            const int32_t* tokens, const uint8_t* mask, int32_t S, int32_t T,
                            int32_t V_total, float* logp, float* lse, float* entropy,
@@ -233,10 +233,10 @@ const char* grpo_status_string(int status);
  * counter. With timing enabled, each launch is bracketed by a pair of CUDA events recorded on
  * its stream (host-side objects; no device memory). */
 enum {
-  GRPO_K_MASK_SCAN = 0, GRPO_K_TILE_LIST, GRPO_K_GROUP_ADV, GRPO_K_FWD_GEMM, GRPO_K_FWD_MERGE,
+  GRPO_K_MASK_SCAN = 0, GRPO_K_PACK, GRPO_K_GROUP_ADV, GRPO_K_FWD_GEMM, GRPO_K_FWD_MERGE,
   GRPO_K_LOSS_TOKENS, GRPO_K_LOSS_FINAL, GRPO_K_BWD_DZ_GEMM, GRPO_K_BWD_DH_GEMM,
-  GRPO_K_BWD_DW_GEMM, GRPO_K_DH_ZERO_TAIL, GRPO_K_F32_FWD, GRPO_K_F32_DH, GRPO_K_F32_DW,
-  GRPO_K_REWARDS, GRPO_K_SHARD_STATS, GRPO_K_MERGE_SHARDS, GRPO_K_COUNT
+  GRPO_K_BWD_DW_GEMM, GRPO_K_DH_ZERO, GRPO_K_F32_FWD, GRPO_K_F32_DH, GRPO_K_F32_DW,
+  GRPO_K_REWARDS, GRPO_K_SHARD_STATS, GRPO_K_MERGE_SHARDS, GRPO_K_GATHER, GRPO_K_COUNT
 };
 const char* grpo_kernel_name(int32_t kernel_id);
 int grpo_timing_enable(int32_t enable);   /* 1 = record events from now on, 0 = stop */

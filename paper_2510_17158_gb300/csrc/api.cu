@@ -19,10 +19,10 @@ namespace {
 // kernel accounting
 // ------------------------------------------------------------------------------------------
 const char* const kKernelNames[GRPO_K_COUNT] = {
-    "mask_scan",       "tile_list",    "group_adv",   "fwd_gemm_tc",  "fwd_merge",
+    "mask_scan",       "pack_tokens",  "group_adv",   "fwd_gemm_tc",  "fwd_merge",
     "loss_tokens",     "loss_final",   "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-    "dh_zero_tail",    "f32_fwd",      "f32_dh",      "f32_dw",      "rewards",
-    "shard_stats",     "merge_shards"};
+    "dh_zero_unscored", "f32_fwd",     "f32_dh",      "f32_dw",      "rewards",
+    "shard_stats",     "merge_shards", "gather_rows"};
 
 struct EventPair {
   cudaEvent_t a, b;
@@ -81,36 +81,40 @@ int counted(int kid, cudaStream_t st, F&& launch) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Layout {
-  int max_tiles;
-  long long rows_cap;
+  int max_tiles;        // packed-row tiles of the worst case (every position scored)
+  long long rows_cap;   // packed-row capacity: S*T rounded up to a multiple of 128
   int num_strips;
   int v_round;          // V rounded up to a multiple of 256
-  size_t seq_last, seq_tile_base, tiles, counts, zy, partials, partials2, g, cvec, seq_loss;
+  size_t seq_base, row_pos, pos_row, counts, zy, partials, partials2, g, cvec, seq_loss, hp, hrp;
   size_t fixed_end;     // end of the regions that do not depend on the vocabulary chunk
 };
 
 Layout make_layout(int S, int T, int d, int V, int dtype) {
-  (void)d;
   Layout L{};
-  L.max_tiles = S * ((T + kTileRows - 1) / kTileRows);
-  L.rows_cap = static_cast<long long>(L.max_tiles) * kTileRows;
+  const size_t P = static_cast<size_t>(S) * T;
+  L.rows_cap = static_cast<long long>((P + kTileRows - 1) / kTileRows) * kTileRows;
+  L.max_tiles = static_cast<int>(L.rows_cap / kTileRows);
   const int nvt = (V + kTileN - 1) / kTileN;
   L.num_strips = (nvt + kFwdTilesPerStrip - 1) / kFwdTilesPerStrip;
   L.v_round = nvt * kTileN;
-  const size_t P = static_cast<size_t>(S) * T;
+  const bool bf16 = dtype == GRPO_BF16;
   size_t off = sizeof(WsHeader);
-  L.seq_last = off;       off = align256(off + sizeof(int32_t) * S);
-  L.seq_tile_base = off;  off = align256(off + sizeof(int32_t) * (S + 1));
-  L.tiles = off;          off = align256(off + sizeof(int2) * L.max_tiles);
+  L.seq_base = off;       off = align256(off + sizeof(int32_t) * (S + 1));
+  L.row_pos = off;        off = align256(off + sizeof(int32_t) * L.rows_cap);
+  L.pos_row = off;        off = align256(off + sizeof(int32_t) * P);
   L.counts = off;         off = align256(off + sizeof(int32_t) * S);
   L.zy = off;             off = align256(off + sizeof(float) * P);
   L.partials = off;
-  if (dtype == GRPO_BF16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  if (bf16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
   L.partials2 = off;      // exact-KL forward only
-  if (dtype == GRPO_BF16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  if (bf16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
   L.g = off;              off = align256(off + sizeof(float) * P);
   L.cvec = off;           off = align256(off + sizeof(float) * P);
   L.seq_loss = off;       off = align256(off + sizeof(float) * S);
+  L.hp = off;             // packed hidden states (bf16 path)
+  if (bf16) off = align256(off + static_cast<size_t>(L.rows_cap) * d * 2);
+  L.hrp = off;            // packed reference hidden states (exact-KL path)
+  if (bf16) off = align256(off + static_cast<size_t>(L.rows_cap) * d * 2);
   L.fixed_end = off;
   return L;
 }
@@ -196,9 +200,9 @@ int gemm_grid(long long row_units, long long col_units, bool pair) {
 
 struct Views {
   WsHeader* hdr;
-  int32_t* seq_last;
-  int32_t* seq_tile_base;
-  int2* tiles;
+  int32_t* seq_base;
+  int32_t* row_pos;
+  int32_t* pos_row;
   int32_t* counts;
   float* zy;
   float4* partials;
@@ -206,15 +210,17 @@ struct Views {
   float* g;
   float* cvec;
   float* seq_loss;
+  void* hp;
+  void* hrp;
 };
 
 Views views(void* ws, const Layout& L) {
   char* b = static_cast<char*>(ws);
   Views v;
   v.hdr = reinterpret_cast<WsHeader*>(b);
-  v.seq_last = reinterpret_cast<int32_t*>(b + L.seq_last);
-  v.seq_tile_base = reinterpret_cast<int32_t*>(b + L.seq_tile_base);
-  v.tiles = reinterpret_cast<int2*>(b + L.tiles);
+  v.seq_base = reinterpret_cast<int32_t*>(b + L.seq_base);
+  v.row_pos = reinterpret_cast<int32_t*>(b + L.row_pos);
+  v.pos_row = reinterpret_cast<int32_t*>(b + L.pos_row);
   v.counts = reinterpret_cast<int32_t*>(b + L.counts);
   v.zy = reinterpret_cast<float*>(b + L.zy);
   v.partials = reinterpret_cast<float4*>(b + L.partials);
@@ -222,8 +228,14 @@ Views views(void* ws, const Layout& L) {
   v.g = reinterpret_cast<float*>(b + L.g);
   v.cvec = reinterpret_cast<float*>(b + L.cvec);
   v.seq_loss = reinterpret_cast<float*>(b + L.seq_loss);
+  v.hp = b + L.hp;
+  v.hrp = b + L.hrp;
   return v;
 }
+
+// Packs the scored tokens: counts from the mask, packed-row maps, and H gathered into Hp.
+int pack_tokens(const uint8_t* mask, int S, int T, int d, const void* H, const Layout& L,
+                const Views& v, int32_t* counts_out, cudaStream_t st);
 
 GemmArgs base_args(const Layout& L, const Views& v, int S, int T, int d, int V,
                    const int32_t* tokens, const uint8_t* mask) {
@@ -233,7 +245,7 @@ GemmArgs base_args(const Layout& L, const Views& v, int S, int T, int d, int V,
   a.T = T;
   a.d = d;
   a.V = V;
-  a.tiles = v.tiles;
+  a.row_pos = v.row_pos;
   a.hdr = v.hdr;
   a.tokens = tokens;
   a.mask = mask;
@@ -241,6 +253,20 @@ GemmArgs base_args(const Layout& L, const Views& v, int S, int T, int d, int V,
   a.num_strips = L.num_strips;
   a.inject_stall = g_inject_stall.load();
   return a;
+}
+
+int pack_tokens(const uint8_t* mask, int S, int T, int d, const void* H, const Layout& L,
+                const Views& v, int32_t* counts_out, cudaStream_t st) {
+  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                   [&] { return launch_mask_scan(mask, S, T, counts_out, st); }));
+  GRPO_TRY(counted(GRPO_K_PACK, st, [&] {
+    return launch_pack(mask, counts_out, S, T, L.rows_cap, v.seq_base, v.row_pos, v.pos_row,
+                       v.hdr, st);
+  }));
+  if (!H) return GRPO_OK;
+  return counted(GRPO_K_GATHER, st, [&] {
+    return launch_gather_rows(H, d, v.row_pos, v.hdr, L.rows_cap, v.hp, st);
+  });
 }
 
 }  // namespace
@@ -323,21 +349,19 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);
 
-  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
-                   [&] { return launch_mask_scan(mask, S, T, valid_count, v.seq_last, st); }));
   if (dtype == GRPO_F32) {
+    GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
+                     [&] { return launch_mask_scan(mask, S, T, valid_count, st); }));
     return counted(GRPO_K_F32_FWD, st, [&] {
       return launch_f32_fwd(static_cast<const float*>(H), static_cast<const float*>(W), tokens,
                             mask, S, T, d, V, logp, lse, entropy, argmax, v.hdr, st);
     });
   }
   if (!aligned16(H) || !aligned16(W)) return GRPO_ERR_INVALID_ARG;
-  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
-    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
-  }));
+  GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, valid_count, st));
   const bool pair = g_cta_pair.load() != 0;
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, H, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapW, W, d, V, d, pair ? kTileN / 2 : kTileN))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
@@ -347,7 +371,7 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   GRPO_TRY(counted(GRPO_K_FWD_GEMM, st,
                    [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st); }));
   return counted(GRPO_K_FWD_MERGE, st, [&] {
-    return launch_fwd_merge(v.partials, L.rows_cap, L.num_strips, v.zy, v.seq_tile_base, tokens,
+    return launch_fwd_merge(v.partials, L.rows_cap, L.num_strips, v.zy, v.pos_row, tokens,
                             mask, S, T, V, logp, lse, entropy, argmax, v.hdr, st);
   });
 }
@@ -396,11 +420,9 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   // ref_logp is not read when beta == 0; pass a valid pointer anyway.
   const float* ref = ref_logp ? ref_logp : logp;
 
-  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
-                   [&] { return launch_mask_scan(mask, S, T, v.counts, v.seq_last, st); }));
-  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
-    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
-  }));
+  // counts from the mask and the packed-row maps (also Sum n for token_mean); H is gathered
+  // below, on the tensor-core path only
+  GRPO_TRY(pack_tokens(mask, S, T, d, nullptr, L, v, v.counts, st));
   GRPO_TRY(counted(GRPO_K_LOSS_TOKENS, st, [&] {
     return launch_loss_tokens(mask, logp, old_logp, ref, adv, valid_count, S, T, eps_low,
                               eps_high, beta, agg, norm, mode, v.hdr, v.g, v.seq_loss, st, kl,
@@ -448,17 +470,24 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     dz = reinterpret_cast<__nv_bfloat16*>(wsb + L.fixed_end +
                                           align256(static_cast<size_t>(L.rows_cap) * d * 4));
   }
+  GRPO_TRY(counted(GRPO_K_GATHER, st, [&] {
+    return launch_gather_rows(H, d, v.row_pos, v.hdr, L.rows_cap, v.hp, st);
+  }));
+  if (mode == 2) {
+    GRPO_TRY(counted(GRPO_K_GATHER, st, [&] {
+      return launch_gather_rows(H_ref, d, v.row_pos, v.hdr, L.rows_cap, v.hrp, st);
+    }));
+  }
   const bool pair = g_cta_pair.load() != 0 && mode != 2;   // exact-KL roles: single-CTA tiles
   CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn, mapHrk, mapWrk;
-  if (mode == 2 && (!make_map(&mapHrk, H_ref, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+  if (mode == 2 && (!make_map(&mapHrk, v.hrp, d, L.rows_cap, d, kTileRows) ||
                     !make_map(&mapWrk, W_ref, d, V, d, kTileN)))
     return GRPO_ERR_CUDA;
-  const uint64_t P = static_cast<uint64_t>(S) * T;
-  if (!make_map(&mapHk, H, d, P, d, kTileRows) ||
+  if (!make_map(&mapHk, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapWk, W, d, V, d, pair ? kTileN / 2 : kTileN) ||
       !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
       !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
-      !make_map(&mapHmn, H, d, P, d, 64))
+      !make_map(&mapHmn, v.hp, d, L.rows_cap, d, 64))
     return GRPO_ERR_CUDA;
 
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
@@ -494,8 +523,8 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
       return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, d / kTileN, pair), pair, st);
     }));
   }
-  return counted(GRPO_K_DH_ZERO_TAIL, st, [&] {
-    return launch_dh_zero_tail(v.seq_tile_base, S, T, d, dH, dh_f32 ? 4 : 2, st);
+  return counted(GRPO_K_DH_ZERO, st, [&] {
+    return launch_dh_zero_masked(mask, S, T, d, dH, dh_f32 ? 4 : 2, st);
   });
 }
 
@@ -543,15 +572,15 @@ int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const voi
   if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);
-  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
-                   [&] { return launch_mask_scan(mask, S, T, valid_count, v.seq_last, st); }));
-  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
-    return launch_tile_list(v.seq_last, valid_count, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
+  GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, valid_count, st));
+  GRPO_TRY(counted(GRPO_K_GATHER, st, [&] {
+    return launch_gather_rows(H_ref, d, v.row_pos, v.hdr, L.rows_cap, v.hrp, st);
   }));
-  const uint64_t P = static_cast<uint64_t>(S) * T;
   CUtensorMap mapH, mapW, mapHr, mapWr;
-  if (!make_map(&mapH, H, d, P, d, kTileRows) || !make_map(&mapW, W, d, V, d, kTileN) ||
-      !make_map(&mapHr, H_ref, d, P, d, kTileRows) || !make_map(&mapWr, W_ref, d, V, d, kTileN))
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
+      !make_map(&mapW, W, d, V, d, kTileN) ||
+      !make_map(&mapHr, v.hrp, d, L.rows_cap, d, kTileRows) ||
+      !make_map(&mapWr, W_ref, d, V, d, kTileN))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
   a.partials = v.partials;
@@ -563,7 +592,7 @@ int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const voi
   }));
   return counted(GRPO_K_FWD_MERGE, st, [&] {
     return launch_fwd_merge_kl(v.partials, v.partials2, L.rows_cap, L.num_strips, v.zy,
-                               v.seq_tile_base, tokens, mask, S, T, V, logp, lse, entropy, argmax,
+                               v.pos_row, tokens, mask, S, T, V, logp, lse, entropy, argmax,
                                lse_ref, kl, v.hdr, st);
   });
 }
@@ -597,14 +626,10 @@ int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
   if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);
-  GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
-                   [&] { return launch_mask_scan(mask, S, T, v.counts, v.seq_last, st); }));
-  GRPO_TRY(counted(GRPO_K_TILE_LIST, st, [&] {
-    return launch_tile_list(v.seq_last, v.counts, S, T, v.seq_tile_base, v.tiles, v.hdr, st);
-  }));
+  GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, v.counts, st));
   const bool pair = g_cta_pair.load() != 0;
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, H, d, static_cast<uint64_t>(S) * T, d, kTileRows) ||
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapW, W_shard, d, V_shard, d, pair ? kTileN / 2 : kTileN))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V_shard, tokens, mask);
@@ -616,7 +641,7 @@ int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
                        st);
   }));
   return counted(GRPO_K_SHARD_STATS, st, [&] {
-    return launch_shard_stats(v.partials, L.rows_cap, L.num_strips, v.zy, v.seq_tile_base, tokens,
+    return launch_shard_stats(v.partials, L.rows_cap, L.num_strips, v.zy, v.pos_row, tokens,
                               mask, S, T, V_shard, v_offset, reinterpret_cast<float4*>(stats), zy,
                               st);
   });
@@ -633,14 +658,13 @@ int grpo_merge_shard_stats(const float* stats, const float* zy, int32_t num_shar
       static_cast<long long>(S) * T >= (1ll << 31))
     return GRPO_ERR_INVALID_ARG;
   if (!aligned16(stats)) return GRPO_ERR_INVALID_ARG;
-  if (!workspace || workspace_bytes < sizeof(WsHeader) + align256(sizeof(int32_t) * S) ||
+  if (!workspace || workspace_bytes < sizeof(WsHeader) ||
       (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return GRPO_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   WsHeader* hdr = static_cast<WsHeader*>(workspace);
-  int32_t* seq_last = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) + sizeof(WsHeader));
   GRPO_TRY(counted(GRPO_K_MASK_SCAN, st,
-                   [&] { return launch_mask_scan(mask, S, T, valid_count, seq_last, st); }));
+                   [&] { return launch_mask_scan(mask, S, T, valid_count, st); }));
   return counted(GRPO_K_MERGE_SHARDS, st, [&] {
     return launch_merge_shards(reinterpret_cast<const float4*>(stats), zy, num_shards, tokens,
                                mask, S, T, V_total, logp, lse, entropy, argmax, hdr, st);

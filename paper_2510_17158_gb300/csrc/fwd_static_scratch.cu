@@ -51,22 +51,25 @@ size_t up256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 struct StaticLayout {
   int max_tiles, num_strips;
   long long rows_cap;
-  size_t seq_last, seq_tile_base, tiles, zy, partials, end;
+  size_t seq_base, row_pos, pos_row, zy, partials, hp, end;
 };
 
-StaticLayout static_layout(int S, int T, int V, int dtype) {
+StaticLayout static_layout(int S, int T, int d, int V, int dtype) {
   StaticLayout L{};
-  L.max_tiles = S * ((T + kTileRows - 1) / kTileRows);
-  L.rows_cap = static_cast<long long>(L.max_tiles) * kTileRows;
+  const size_t P = static_cast<size_t>(S) * T;
+  L.rows_cap = static_cast<long long>((P + kTileRows - 1) / kTileRows) * kTileRows;
+  L.max_tiles = static_cast<int>(L.rows_cap / kTileRows);
   const int nvt = (V + kTileN - 1) / kTileN;
   L.num_strips = (nvt + kFwdTilesPerStrip - 1) / kFwdTilesPerStrip;
   size_t off = sizeof(WsHeader);
-  L.seq_last = off;      off = up256(off + sizeof(int32_t) * S);
-  L.seq_tile_base = off; off = up256(off + sizeof(int32_t) * (S + 1));
-  L.tiles = off;         off = up256(off + sizeof(int2) * L.max_tiles);
-  L.zy = off;            off = up256(off + sizeof(float) * static_cast<size_t>(S) * T);
+  L.seq_base = off;      off = up256(off + sizeof(int32_t) * (S + 1));
+  L.row_pos = off;       off = up256(off + sizeof(int32_t) * L.rows_cap);
+  L.pos_row = off;       off = up256(off + sizeof(int32_t) * P);
+  L.zy = off;            off = up256(off + sizeof(float) * P);
   L.partials = off;
   if (dtype == GRPO_BF16) off = up256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  L.hp = off;
+  if (dtype == GRPO_BF16) off = up256(off + static_cast<size_t>(L.rows_cap) * d * 2);
   L.end = off;
   return L;
 }
@@ -121,7 +124,7 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
   } else {
     return GRPO_ERR_INVALID_ARG;
   }
-  const StaticLayout L = static_layout(S, T, V, dtype);
+  const StaticLayout L = static_layout(S, T, d, V, dtype);
   if (L.end > kStaticScratchBytes) return GRPO_ERR_WORKSPACE;  // batch too large for the array
 
   void* base = nullptr;
@@ -129,28 +132,32 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
   if (st_addr != GRPO_OK) return st_addr;
   char* b = static_cast<char*>(base);
   WsHeader* hdr = reinterpret_cast<WsHeader*>(b);
-  int32_t* seq_last = reinterpret_cast<int32_t*>(b + L.seq_last);
-  int32_t* seq_tile_base = reinterpret_cast<int32_t*>(b + L.seq_tile_base);
-  int2* tiles = reinterpret_cast<int2*>(b + L.tiles);
+  int32_t* seq_base = reinterpret_cast<int32_t*>(b + L.seq_base);
+  int32_t* row_pos = reinterpret_cast<int32_t*>(b + L.row_pos);
+  int32_t* pos_row = reinterpret_cast<int32_t*>(b + L.pos_row);
   float* zy = reinterpret_cast<float*>(b + L.zy);
   float4* partials = reinterpret_cast<float4*>(b + L.partials);
+  void* hp = b + L.hp;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
 
   // The array keeps the previous call's contents: the status word must start at zero. Every
   // other region used below is fully written before it is read within this call.
   int rc = ok_or_cuda(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), st));
   if (rc != GRPO_OK) return rc;
-  rc = ok_or_cuda(launch_mask_scan(mask, S, T, valid_count, seq_last, st));
+  rc = ok_or_cuda(launch_mask_scan(mask, S, T, valid_count, st));
   if (rc != GRPO_OK) return rc;
   if (dtype == GRPO_F32) {
     rc = ok_or_cuda(launch_f32_fwd(static_cast<const float*>(H), static_cast<const float*>(W),
                                    tokens, mask, S, T, d, V, logp, lse, entropy, argmax, hdr, st));
   } else {
-    rc = ok_or_cuda(launch_tile_list(seq_last, valid_count, S, T, seq_tile_base, tiles, hdr, st));
+    rc = ok_or_cuda(launch_pack(mask, valid_count, S, T, L.rows_cap, seq_base, row_pos, pos_row,
+                                hdr, st));
+    if (rc != GRPO_OK) return rc;
+    rc = ok_or_cuda(launch_gather_rows(H, d, row_pos, hdr, L.rows_cap, hp, st));
     if (rc != GRPO_OK) return rc;
     const bool pair = gemm_pair_mode();
     CUtensorMap mapH, mapW;
-    if (!bf16_map(&mapH, H, d, static_cast<uint64_t>(S) * T, kTileRows) ||
+    if (!bf16_map(&mapH, hp, d, static_cast<uint64_t>(L.rows_cap), kTileRows) ||
         !bf16_map(&mapW, W, d, V, pair ? kTileN / 2 : kTileN))
       return GRPO_ERR_CUDA;
     GemmArgs a;
@@ -159,7 +166,7 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     a.T = T;
     a.d = d;
     a.V = V;
-    a.tiles = tiles;
+    a.row_pos = row_pos;
     a.hdr = hdr;
     a.tokens = tokens;
     a.mask = mask;
@@ -182,7 +189,7 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     }
     rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st));
     if (rc != GRPO_OK) return rc;
-    rc = ok_or_cuda(launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, seq_tile_base,
+    rc = ok_or_cuda(launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, pos_row,
                                      tokens, mask, S, T, V, logp, lse, entropy, argmax, hdr, st));
   }
   if (rc != GRPO_OK) return rc;

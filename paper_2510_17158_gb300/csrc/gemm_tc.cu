@@ -151,11 +151,7 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
     decode_unit(u, sc.num_mu, dm.num_n, mu, n);
     sc.m_of(mu, dm.num_m, m, m_load, m_ok);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n);
-    int hrow = 0;
-    if (ROLE == ROLE_FWD || ROLE == ROLE_DZ || Dual<ROLE>::value) {
-      const int2 tl = a.tiles[m_load];
-      hrow = tl.x * a.T + tl.y;
-    }
+    const int hrow = m_load * BM;   // first packed row of the tile (FWD / DZ / KL A operand)
     for (int t = 0; t < nacc && ok; ++t) {
       for (int kb = 0; kb < dm.num_kb; ++kb) {
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, a.hdr,
@@ -200,8 +196,7 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
 #pragma unroll
             for (int j = 0; j < BM / 64; ++j)
               load(dA + j * BOX_MN, mapA, m_load * BM + j * 64, kb * BK);
-            const int2 tl = a.tiles[kb >> 1];
-            const int row = tl.x * a.T + tl.y + (kb & 1) * BK;
+            const int row = kb * BK;    // K runs over packed rows
 #pragma unroll
             for (int j = 0; j < B_BOXES; ++j)
               load(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, row);
@@ -368,9 +363,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
     sc.m_of(mu, dm.num_m, m, m_load, m_ok);
 
     if (ROLE == ROLE_FWD) {
-      const int2 tl = a.tiles[m_load];
-      const bool rv = m_ok && tl.y + r < a.T;
-      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
+      const bool rv = m_ok && prow >= 0;
+      const long long pos = rv ? prow : 0;
       // sampled token as a column of this W (a vocabulary shard's rows start at v_offset)
       const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] - a.v_offset : -1;
       float rm = -INFINITY, rs = 0.f, ru = 0.f, zyv = 0.f;
@@ -439,9 +434,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
 
     } else if (ROLE == ROLE_FWD_KL) {
       // policy z in columns 0-255, reference z_ref in 256-511 of the one buffer
-      const int2 tl = a.tiles[m_load];
-      const bool rv = m_ok && tl.y + r < a.T;
-      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
+      const bool rv = m_ok && prow >= 0;
+      const long long pos = rv ? prow : 0;
       const int y = (rv && a.mask[pos] != 0) ? a.tokens[pos] : -1;
       float rm = -INFINITY, rs = 0.f, ru = 0.f, rc = 0.f, zyv = 0.f;
       float qm = -INFINITY, qs = 0.f;
@@ -526,9 +521,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
 
     } else if (ROLE == ROLE_DZ_KL) {
       // dz = g (onehot - p) + c p (log p - log q - KL), p from z, q from z_ref
-      const int2 tl = a.tiles[m_load];
-      const bool rv = m_ok && tl.y + r < a.T;
-      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
+      const bool rv = m_ok && prow >= 0;
+      const long long pos = rv ? prow : 0;
       const bool act = rv && a.mask[pos] != 0;
       const float gt = act ? a.g[pos] : 0.f;
       const float ct = act ? a.c[pos] : 0.f;
@@ -576,9 +571,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       bphase ^= 1u;
 
     } else if (ROLE == ROLE_DZ) {
-      const int2 tl = a.tiles[m_load];
-      const bool rv = m_ok && tl.y + r < a.T;
-      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
+      const bool rv = m_ok && prow >= 0;
+      const long long pos = rv ? prow : 0;
       const bool act = rv && a.mask[pos] != 0;
       const float gt = act ? a.g[pos] : 0.f;
       const float ll = act ? a.lse[pos] * kLog2e : 0.f;
@@ -618,9 +613,9 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       if (buf == 0) bphase ^= 1u;
 
     } else if (ROLE == ROLE_DH) {
-      const int2 tl = a.tiles[m_load];
-      const bool rv = m_ok && tl.y + r < a.T;
-      const long long pos = static_cast<long long>(tl.x) * a.T + tl.y + r;
+      const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
+      const bool rv = m_ok && prow >= 0;
+      const long long pos = rv ? prow : 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
       for (int c = 0; c < BN / 32; ++c) {

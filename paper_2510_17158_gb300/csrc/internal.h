@@ -11,9 +11,9 @@ namespace grpo {
 
 struct WsHeader;
 
-// Token tiles: 128 consecutive positions of one sequence, (seq, t0). Tiles of a sequence cover
-// positions 0 .. last scored position; tile k occupies rows k*128 .. k*128+127 of "tile space",
-// the compact row numbering used by the dz scratch and by the GEMMs.
+// Packed rows: the scored tokens of all sequences, in order, numbered 0 .. N-1 (then padded to a
+// multiple of 128). The GEMMs run 128-row tiles over packed rows; the dz scratch, the dH
+// accumulator and the forward partials are indexed by packed row.
 constexpr int kTileRows = 128;
 // Vocabulary tile (N of the forward and dz GEMMs) and hidden tile (N of the dH / dW GEMMs).
 constexpr int kTileN = 256;
@@ -29,11 +29,11 @@ enum GemmRole : int {
 // Arguments of the tcgen05 GEMM kernels (one struct for the four roles).
 struct GemmArgs {
   int S, T, d, V;
-  const int2* tiles;        // [max_tiles] (seq, t0)
+  const int32_t* row_pos;   // [rows_cap] packed row -> position (-1 for padding rows)
   WsHeader* hdr;            // num_tiles, status word
   const int32_t* tokens;    // [S*T]
   const uint8_t* mask;      // [S*T]
-  long long rows_cap;       // max_tiles * 128
+  long long rows_cap;       // packed-row capacity: S*T rounded up to a multiple of 128
   // vocabulary chunk (DZ / DH / DW)
   int vc0, vc_len, dz_pitch;
   // FWD: partial statistics per (strip, tile row) and the target logit per position
@@ -67,14 +67,21 @@ struct GemmArgs {
 
 // Launches (all asynchronous on `st`; return the cudaError_t of the launch).
 cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
-                             int32_t* seq_last, cudaStream_t st);
-cudaError_t launch_tile_list(const int32_t* seq_last, const int32_t* counts, int S, int T,
-                             int32_t* seq_tile_base, int2* tiles, WsHeader* hdr, cudaStream_t st);
+                             cudaStream_t st);
+// Token packing: counts -> seq_base [S+1] (prefix), header (num_tiles = packed rows / 128,
+// total_valid), row_pos [rows_cap] (packed row -> position, -1 for padding) and pos_row [S*T]
+// (position -> packed row, -1 if unscored).
+cudaError_t launch_pack(const uint8_t* mask, const int32_t* counts, int S, int T,
+                        long long rows_cap, int32_t* seq_base, int32_t* row_pos, int32_t* pos_row,
+                        WsHeader* hdr, cudaStream_t st);
+// Hp [packed rows, d] = H rows at row_pos (bf16), zero for padding rows.
+cudaError_t launch_gather_rows(const void* H, int d, const int32_t* row_pos, const WsHeader* hdr,
+                               long long rows_cap, void* Hp, cudaStream_t st);
 cudaError_t launch_group_adv(const float* rewards, const int32_t* go, int num_groups, int S,
                              int std_mode, float std_eps, float* adv, WsHeader* hdr,
                              cudaStream_t st);
 cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num_strips,
-                             const float* zy, const int32_t* seq_tile_base,
+                             const float* zy, const int32_t* pos_row,
                              const int32_t* tokens, const uint8_t* mask, int S, int T, int V,
                              float* logp, float* lse, float* entropy, int32_t* argmax,
                              WsHeader* hdr, cudaStream_t st);
@@ -88,7 +95,7 @@ cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const flo
                                const float* kl = nullptr, float* c = nullptr);
 cudaError_t launch_fwd_merge_kl(const float4* partials, const float4* partials2,
                                 long long rows_cap, int num_strips, const float* zy,
-                                const int32_t* seq_tile_base, const int32_t* tokens,
+                                const int32_t* pos_row, const int32_t* tokens,
                                 const uint8_t* mask, int S, int T, int V, float* logp, float* lse,
                                 float* entropy, int32_t* argmax, float* lse_ref, float* kl,
                                 WsHeader* hdr, cudaStream_t st);
@@ -97,10 +104,10 @@ cudaError_t launch_rewards(const uint8_t* correct, const float* t_base, const fl
                            float* r, cudaStream_t st);
 cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm,
                               const WsHeader* hdr, float* loss_out, cudaStream_t st);
-cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d, void* dH,
-                                int elem_bytes, cudaStream_t st);
+cudaError_t launch_dh_zero_masked(const uint8_t* mask, int S, int T, int d, void* dH,
+                                  int elem_bytes, cudaStream_t st);
 cudaError_t launch_shard_stats(const float4* partials, long long rows_cap, int num_strips,
-                               const float* zy_ws, const int32_t* seq_tile_base,
+                               const float* zy_ws, const int32_t* pos_row,
                                const int32_t* tokens, const uint8_t* mask, int S, int T,
                                int V_shard, int v_offset, float4* stats, float* zy_out,
                                cudaStream_t st);

@@ -23,96 +23,146 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // ------------------------------------------------------------------------------------------
-// Valid counts n_i and the last scored position + 1 of every sequence (one warp per sequence).
+// Valid counts n_i of every sequence (one warp per sequence).
 // ------------------------------------------------------------------------------------------
 __global__ void k_mask_scan(const uint8_t* __restrict__ mask, int S, int T,
-                            int32_t* __restrict__ counts, int32_t* __restrict__ seq_last) {
+                            int32_t* __restrict__ counts) {
   const int warps = blockDim.x / 32;
   const int i = blockIdx.x * warps + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
   if (i >= S) return;
   const uint8_t* row = mask + static_cast<size_t>(i) * T;
-  int cnt = 0, last = 0;
-  for (int t = lane; t < T; t += 32) {
-    if (row[t] != 0) {
-      ++cnt;
-      last = t + 1;
-    }
-  }
+  int cnt = 0;
+  for (int t = lane; t < T; t += 32) cnt += (row[t] != 0);
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    cnt += __shfl_xor_sync(kFull, cnt, o);
-    last = max(last, __shfl_xor_sync(kFull, last, o));
-  }
-  if (lane == 0) {
-    counts[i] = cnt;
-    seq_last[i] = last;
-  }
+  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+  if (lane == 0) counts[i] = cnt;
 }
 
 // ------------------------------------------------------------------------------------------
-// Tile list: sequence i gets ceil(last_i / 128) tiles; exclusive prefix over sequences in one
-// block of 1024 threads (chunks of 1024 sequences, carried).
+// Token packing. The scored tokens of all sequences, in order, become consecutive "packed rows"
+// (sequence i's tokens start at seq_base[i] = n_0 + ... + n_{i-1}); the GEMMs run 128-row tiles
+// over packed rows, so no tile row is spent on padding or on masked (tool-result) tokens.
+// k_seq_scan: exclusive prefix of the counts (one block of 1024, chunks of 1024 carried), total
+// and tile count into the header, and row_pos = -1 for the padding rows of the last tile.
 // ------------------------------------------------------------------------------------------
-__global__ void k_tile_list(const int32_t* __restrict__ seq_last, const int32_t* __restrict__ counts,
-                            int S, int T, int32_t* __restrict__ seq_tile_base,
-                            int2* __restrict__ tiles, WsHeader* hdr) {
-  __shared__ int warp_tot[32];
-  __shared__ long long warp_cnt[32];
-  __shared__ int carry_s;
-  __shared__ long long carry_c;
+__global__ void k_seq_scan(const int32_t* __restrict__ counts, int S, long long rows_cap,
+                           int32_t* __restrict__ seq_base, int32_t* __restrict__ row_pos,
+                           WsHeader* hdr) {
+  __shared__ long long warp_tot[32];
+  __shared__ long long carry;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  if (tid == 0) {
-    carry_s = 0;
-    carry_c = 0;
-  }
+  if (tid == 0) carry = 0;
   __syncthreads();
   for (int base = 0; base < S; base += 1024) {
     const int i = base + tid;
-    const int nt = (i < S) ? (seq_last[i] + kTileRows - 1) / kTileRows : 0;
-    const long long nc = (i < S) ? counts[i] : 0;
-    // inclusive warp scan of nt
-    int x = nt;
+    const long long n = (i < S) ? counts[i] : 0;
+    long long x = n;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int y = __shfl_up_sync(kFull, x, o);
+      const long long y = __shfl_up_sync(kFull, x, o);
       if (lane >= o) x += y;
     }
-    long long c = nc;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFull, c, o);
     if (lane == 31) warp_tot[wid] = x;
-    if (lane == 0) warp_cnt[wid] = c;
     __syncthreads();
     if (wid == 0) {
-      int w = warp_tot[lane];
-      int xs = w;
+      const long long w = warp_tot[lane];
+      long long xs = w;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        int y = __shfl_up_sync(kFull, xs, o);
+        const long long y = __shfl_up_sync(kFull, xs, o);
         if (lane >= o) xs += y;
       }
-      warp_tot[lane] = xs - w;  // exclusive prefix of warp totals
+      warp_tot[lane] = xs - w;
     }
     __syncthreads();
-    const int excl = carry_s + warp_tot[wid] + x - nt;
-    if (i < S) {
-      seq_tile_base[i] = excl;
-      for (int k = 0; k < nt; ++k) tiles[excl + k] = make_int2(i, k * kTileRows);
-    }
+    const long long excl = carry + warp_tot[wid] + x - n;
+    if (i < S) seq_base[i] = static_cast<int32_t>(excl);
     __syncthreads();
-    if (tid == 1023) carry_s = excl + nt;
-    if (tid == 0) {
-      long long s = 0;
-      for (int w = 0; w < 32; ++w) s += warp_cnt[w];
-      carry_c += s;
-    }
+    if (tid == 1023) carry = excl + n;
     __syncthreads();
   }
+  const long long total = carry;
+  const long long padded = (total + kTileRows - 1) / kTileRows * kTileRows;
+  for (long long r = total + tid; r < padded && r < rows_cap; r += blockDim.x) row_pos[r] = -1;
   if (tid == 0) {
-    seq_tile_base[S] = carry_s;
-    hdr->num_tiles = carry_s;
-    hdr->total_valid = carry_c;
+    seq_base[S] = static_cast<int32_t>(total);
+    hdr->num_tiles = static_cast<int32_t>(padded / kTileRows);
+    hdr->total_valid = total;
+  }
+}
+
+// One block per sequence: ranks of the scored positions (block-wide scan over T), and the two
+// maps packed row -> position (row_pos) and position -> packed row (pos_row, -1 if unscored).
+constexpr int kPackThreads = 256;
+
+__global__ void __launch_bounds__(kPackThreads)
+    k_pack(const uint8_t* __restrict__ mask, int S, int T, const int32_t* __restrict__ seq_base,
+           int32_t* __restrict__ row_pos, int32_t* __restrict__ pos_row) {
+  __shared__ int warp_tot[kPackThreads / 32];
+  const int i = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int chunk = (T + kPackThreads - 1) / kPackThreads;
+  const int t0 = min(T, tid * chunk), t1 = min(T, t0 + chunk);
+  const size_t rowb = static_cast<size_t>(i) * T;
+  int n = 0;
+  for (int t = t0; t < t1; ++t) n += (mask[rowb + t] != 0);
+  int x = n;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    const int w = lane < kPackThreads / 32 ? warp_tot[lane] : 0;
+    int xs = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, xs, o);
+      if (lane >= o) xs += y;
+    }
+    if (lane < kPackThreads / 32) warp_tot[lane] = xs - w;
+  }
+  __syncthreads();
+  int r = seq_base[i] + warp_tot[wid] + x - n;
+  for (int t = t0; t < t1; ++t) {
+    const size_t pos = rowb + t;
+    if (mask[pos] != 0) {
+      row_pos[r] = static_cast<int32_t>(pos);
+      pos_row[pos] = r;
+      ++r;
+    } else {
+      pos_row[pos] = -1;
+    }
+  }
+}
+
+// Hp[r, :] = H[row_pos[r], :] for the packed rows of the current batch (zero for padding rows).
+__global__ void k_gather_rows(const uint4* __restrict__ H, int vec_per_row,
+                              const int32_t* __restrict__ row_pos, const WsHeader* hdr,
+                              uint4* __restrict__ Hp) {
+  const long long rows = static_cast<long long>(hdr->num_tiles) * kTileRows;
+  for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
+    const int pos = row_pos[r];
+    uint4* dst = Hp + r * vec_per_row;
+    if (pos >= 0) {
+      const uint4* src = H + static_cast<long long>(pos) * vec_per_row;
+      for (int k = threadIdx.x; k < vec_per_row; k += blockDim.x) dst[k] = src[k];
+    } else {
+      for (int k = threadIdx.x; k < vec_per_row; k += blockDim.x) dst[k] = make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+
+// dH rows of unscored positions are zero (scored rows are written by the dH GEMM).
+__global__ void k_dh_zero_masked(const uint8_t* __restrict__ mask, long long P, int vec_per_row,
+                                 uint4* __restrict__ dH) {
+  for (long long pos = blockIdx.x; pos < P; pos += gridDim.x) {
+    if (mask[pos] != 0) continue;
+    uint4* p = dH + pos * vec_per_row;
+    for (int k = threadIdx.x; k < vec_per_row; k += blockDim.x) p[k] = make_uint4(0, 0, 0, 0);
   }
 }
 
@@ -167,7 +217,7 @@ __global__ void k_group_adv(const float* __restrict__ r, const int32_t* __restri
 // ------------------------------------------------------------------------------------------
 __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_cap,
                             int num_strips, const float* __restrict__ zy,
-                            const int32_t* __restrict__ seq_tile_base,
+                            const int32_t* __restrict__ pos_row,
                             const int32_t* __restrict__ tokens, const uint8_t* __restrict__ mask,
                             int S, int T, int V, float* __restrict__ logp,
                             float* __restrict__ lse_out, float* __restrict__ entropy,
@@ -181,9 +231,7 @@ __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_
     argmax[pos] = -1;
     return;
   }
-  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
-  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
-                        (t % kTileRows);
+  const long long row = pos_row[pos];   // packed row of this scored position
   float M = -INFINITY;
   int idx = 0;
   for (int j = 0; j < num_strips; ++j) {
@@ -220,7 +268,7 @@ __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_
 __global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
                                const float4* __restrict__ partials2, long long rows_cap,
                                int num_strips, const float* __restrict__ zy,
-                               const int32_t* __restrict__ seq_tile_base,
+                               const int32_t* __restrict__ pos_row,
                                const int32_t* __restrict__ tokens,
                                const uint8_t* __restrict__ mask, int S, int T, int V,
                                float* __restrict__ logp, float* __restrict__ lse_out,
@@ -238,9 +286,7 @@ __global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
     kl[pos] = 0.f;
     return;
   }
-  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
-  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
-                        (t % kTileRows);
+  const long long row = pos_row[pos];   // packed row of this scored position
   float M = -INFINITY, Mr = -INFINITY;
   int idx = 0;
   for (int j = 0; j < num_strips; ++j) {
@@ -392,30 +438,12 @@ __global__ void k_loss_final(const float* __restrict__ seq_loss, int S, float* l
 }
 
 // ------------------------------------------------------------------------------------------
-// dH rows that no token tile covers (positions after a sequence's last tile) are zero.
-// ------------------------------------------------------------------------------------------
-__global__ void k_dh_zero_tail(const int32_t* __restrict__ seq_tile_base, int S, int T, int d,
-                               char* __restrict__ dH, int elem_bytes) {
-  const int tb = blockIdx.x, i = blockIdx.y;
-  const int covered = seq_tile_base[i + 1] - seq_tile_base[i];
-  if (tb < covered) return;
-  const int t0 = tb * kTileRows;
-  const int t1 = min(T, t0 + kTileRows);
-  if (t0 >= t1) return;
-  const size_t beg = (static_cast<size_t>(i) * T + t0) * d * elem_bytes;
-  const size_t n = static_cast<size_t>(t1 - t0) * d * elem_bytes / 2;  // d % 64 == 0
-  uint4* p = reinterpret_cast<uint4*>(dH + beg);
-  const uint4 z = make_uint4(0, 0, 0, 0);
-  for (size_t k = threadIdx.x; k < n / 8; k += blockDim.x) p[k] = z;
-}
-
-// ------------------------------------------------------------------------------------------
 // Vocabulary-parallel scoring: statistics of one shard per position, and the merge of the
 // statistics of all shards.
 // ------------------------------------------------------------------------------------------
 __global__ void k_shard_stats(const float4* __restrict__ partials, long long rows_cap,
                               int num_strips, const float* __restrict__ zy_ws,
-                              const int32_t* __restrict__ seq_tile_base,
+                              const int32_t* __restrict__ pos_row,
                               const int32_t* __restrict__ tokens,
                               const uint8_t* __restrict__ mask, int S, int T, int V_shard,
                               int v_offset, float4* __restrict__ stats,
@@ -427,9 +455,7 @@ __global__ void k_shard_stats(const float4* __restrict__ partials, long long row
     zy_out[pos] = -INFINITY;
     return;
   }
-  const int i = static_cast<int>(pos / T), t = static_cast<int>(pos % T);
-  const long long row = static_cast<long long>(seq_tile_base[i] + t / kTileRows) * kTileRows +
-                        (t % kTileRows);
+  const long long row = pos_row[pos];   // packed row of this scored position
   float M = -INFINITY;
   int idx = 0;
   for (int j = 0; j < num_strips; ++j) {
@@ -691,15 +717,38 @@ __global__ void __launch_bounds__(kF32Threads)
 // launches
 // ------------------------------------------------------------------------------------------
 cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
-                             int32_t* seq_last, cudaStream_t st) {
+                             cudaStream_t st) {
   const int warps = 8;
-  k_mask_scan<<<(S + warps - 1) / warps, warps * 32, 0, st>>>(mask, S, T, counts, seq_last);
+  k_mask_scan<<<(S + warps - 1) / warps, warps * 32, 0, st>>>(mask, S, T, counts);
   return cudaGetLastError();
 }
 
-cudaError_t launch_tile_list(const int32_t* seq_last, const int32_t* counts, int S, int T,
-                             int32_t* seq_tile_base, int2* tiles, WsHeader* hdr, cudaStream_t st) {
-  k_tile_list<<<1, 1024, 0, st>>>(seq_last, counts, S, T, seq_tile_base, tiles, hdr);
+cudaError_t launch_pack(const uint8_t* mask, const int32_t* counts, int S, int T,
+                        long long rows_cap, int32_t* seq_base, int32_t* row_pos, int32_t* pos_row,
+                        WsHeader* hdr, cudaStream_t st) {
+  k_seq_scan<<<1, 1024, 0, st>>>(counts, S, rows_cap, seq_base, row_pos, hdr);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_pack<<<S, kPackThreads, 0, st>>>(mask, S, T, seq_base, row_pos, pos_row);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_rows(const void* H, int d, const int32_t* row_pos, const WsHeader* hdr,
+                               long long rows_cap, void* Hp, cudaStream_t st) {
+  const int vec = d * 2 / 16;                 // bf16 rows, d % 64 == 0
+  const long long blocks = rows_cap < 8192 ? (rows_cap > 0 ? rows_cap : 1) : 8192;
+  k_gather_rows<<<static_cast<unsigned>(blocks), 128, 0, st>>>(
+      static_cast<const uint4*>(H), vec, row_pos, hdr, static_cast<uint4*>(Hp));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dh_zero_masked(const uint8_t* mask, int S, int T, int d, void* dH,
+                                  int elem_bytes, cudaStream_t st) {
+  const long long P = static_cast<long long>(S) * T;
+  const int vec = d * elem_bytes / 16;
+  const long long blocks = P < 16384 ? (P > 0 ? P : 1) : 16384;
+  k_dh_zero_masked<<<static_cast<unsigned>(blocks), 128, 0, st>>>(mask, P, vec,
+                                                                  static_cast<uint4*>(dH));
   return cudaGetLastError();
 }
 
@@ -711,14 +760,14 @@ cudaError_t launch_group_adv(const float* rewards, const int32_t* go, int num_gr
 }
 
 cudaError_t launch_fwd_merge(const float4* partials, long long rows_cap, int num_strips,
-                             const float* zy, const int32_t* seq_tile_base,
+                             const float* zy, const int32_t* pos_row,
                              const int32_t* tokens, const uint8_t* mask, int S, int T, int V,
                              float* logp, float* lse, float* entropy, int32_t* argmax,
                              WsHeader* hdr, cudaStream_t st) {
   const long long P = static_cast<long long>(S) * T;
   const int threads = 256;
   k_fwd_merge<<<static_cast<unsigned>((P + threads - 1) / threads), threads, 0, st>>>(
-      partials, rows_cap, num_strips, zy, seq_tile_base, tokens, mask, S, T, V, logp, lse,
+      partials, rows_cap, num_strips, zy, pos_row, tokens, mask, S, T, V, logp, lse,
       entropy, argmax, hdr);
   return cudaGetLastError();
 }
@@ -737,13 +786,13 @@ cudaError_t launch_loss_tokens(const uint8_t* mask, const float* logp, const flo
 
 cudaError_t launch_fwd_merge_kl(const float4* partials, const float4* partials2,
                                 long long rows_cap, int num_strips, const float* zy,
-                                const int32_t* seq_tile_base, const int32_t* tokens,
+                                const int32_t* pos_row, const int32_t* tokens,
                                 const uint8_t* mask, int S, int T, int V, float* logp, float* lse,
                                 float* entropy, int32_t* argmax, float* lse_ref, float* kl,
                                 WsHeader* hdr, cudaStream_t st) {
   const long long P = static_cast<long long>(S) * T;
   k_fwd_merge_kl<<<static_cast<unsigned>((P + 255) / 256), 256, 0, st>>>(
-      partials, partials2, rows_cap, num_strips, zy, seq_tile_base, tokens, mask, S, T, V, logp,
+      partials, partials2, rows_cap, num_strips, zy, pos_row, tokens, mask, S, T, V, logp,
       lse, entropy, argmax, lse_ref, kl, hdr);
   return cudaGetLastError();
 }
@@ -765,22 +814,14 @@ cudaError_t launch_loss_final(const float* seq_loss, int S, int agg, double norm
   return cudaGetLastError();
 }
 
-cudaError_t launch_dh_zero_tail(const int32_t* seq_tile_base, int S, int T, int d, void* dH,
-                                int elem_bytes, cudaStream_t st) {
-  dim3 grid((T + kTileRows - 1) / kTileRows, S);
-  k_dh_zero_tail<<<grid, 256, 0, st>>>(seq_tile_base, S, T, d, static_cast<char*>(dH),
-                                       elem_bytes);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_shard_stats(const float4* partials, long long rows_cap, int num_strips,
-                               const float* zy_ws, const int32_t* seq_tile_base,
+                               const float* zy_ws, const int32_t* pos_row,
                                const int32_t* tokens, const uint8_t* mask, int S, int T,
                                int V_shard, int v_offset, float4* stats, float* zy_out,
                                cudaStream_t st) {
   const long long P = static_cast<long long>(S) * T;
   k_shard_stats<<<static_cast<unsigned>((P + 255) / 256), 256, 0, st>>>(
-      partials, rows_cap, num_strips, zy_ws, seq_tile_base, tokens, mask, S, T, V_shard,
+      partials, rows_cap, num_strips, zy_ws, pos_row, tokens, mask, S, T, V_shard,
       v_offset, stats, zy_out);
   return cudaGetLastError();
 }

@@ -25,10 +25,10 @@ AGG_MODES = {"seq_mean": 0, "token_mean": 1}
 STATUS_NAMES = {0: "GRPO_OK", -1: "GRPO_ERR_INVALID_ARG", -2: "GRPO_ERR_UNSUPPORTED",
                 -3: "GRPO_ERR_CUDA", -4: "GRPO_ERR_WORKSPACE", -5: "GRPO_ERR_TOKEN_RANGE",
                 -6: "GRPO_ERR_TIMEOUT", -7: "GRPO_ERR_GROUPS"}
-KERNEL_NAMES = ["mask_scan", "tile_list", "group_adv", "fwd_gemm_tc", "fwd_merge", "loss_tokens",
+KERNEL_NAMES = ["mask_scan", "pack_tokens", "group_adv", "fwd_gemm_tc", "fwd_merge", "loss_tokens",
                 "loss_final", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc",
-                "dh_zero_tail", "f32_fwd", "f32_dh", "f32_dw", "rewards", "shard_stats",
-                "merge_shards"]
+                "dh_zero_unscored", "f32_fwd", "f32_dh", "f32_dw", "rewards", "shard_stats",
+                "merge_shards", "gather_rows"]
 
 
 class GrpoError(RuntimeError):
