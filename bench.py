@@ -273,6 +273,16 @@ def run_gpu(args):
     dev_args = (b.H, b.W, b.tokens, b.mask, b.rewards, b.group_offsets, old, ref)
     for _ in range(args.warmup):
         step(*dev_args)
+    graph = None
+    launches_per_graph = 0
+    if args.graph:      # the whole step as one CUDA graph (all launches replayed at once)
+        torch.cuda.synchronize()
+        G.grpo_timing_reset()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step(*dev_args)
+        launches_per_graph = sum(n for n, _ in G.timing_table().values())
+        graph.replay()
     torch.cuda.synchronize()
     st, where = G.grpo_last_device_error(ws)
     if st != 0:
@@ -287,7 +297,10 @@ def run_gpu(args):
         torch.cuda.synchronize()
         ev0.record(stream)
         for _ in range(args.steps):
-            step(*dev_args)
+            if graph is not None:
+                graph.replay()
+            else:
+                step(*dev_args)
         ev1.record(stream)
         torch.cuda.synchronize()
         barrier(ws_n)
@@ -296,6 +309,8 @@ def run_gpu(args):
     ms_max = dist_max(ms, ws_n, device)
     table = G.timing_table()
     launches = sum(n for n, _ in table.values())
+    if graph is not None:    # replays record no per-kernel events; launches come from the capture
+        launches = launches_per_graph * args.steps
     st, where = G.grpo_last_device_error(ws)
     if st != 0:
         raise RuntimeError(f"device status {st} at {where} in the timed region")
@@ -354,6 +369,8 @@ def run_gpu(args):
     # ---- roofline of the dominant kernel -------------------------------------------------------
     per_kernel = {k: {"launches": n, "ms_total": round(t, 3), "ms_per_launch": round(t / n, 4),
                       "share": round(t / ms, 4)} for k, (n, t) in table.items()}
+    if not table:            # graph replays: no per-kernel timing
+        table = {"graph_replay": (args.steps, ms)}
     dom = max(table, key=lambda k: table[k][1])
     n_dom, t_dom = table[dom]
     chunk = args.vocab_chunk or V
@@ -391,7 +408,8 @@ def run_gpu(args):
                             "single CTA 128x256 (cta_group::1)",
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
                        b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
-                   "parallelism": f"dp{ws_n} (independent groups per GPU)"},
+                   "parallelism": f"dp{ws_n} (independent groups per GPU)",
+                   "cuda_graph": bool(args.graph)},
         "tflops_alg": round(alg_tflops, 1),
         "frac_of_bf16_peak": round(alg_tflops / pk["bf16"], 4),
         "frac_of_bf16_sustained": round(alg_tflops / pk["bf16_sustained"], 4),
@@ -431,6 +449,9 @@ def main():
                          "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
     ap.add_argument("--cta-pair", type=int, default=0,
                     help="tensor-core tiles: 0 = single CTAs (default), 1 = CTA pairs (cta_group::2)")
+    ap.add_argument("--graph", action="store_true",
+                    help="capture one step in a CUDA graph and time its replays (per-kernel "
+                         "timing and launch counts then come from the capture, not the replays)")
     ap.add_argument("--scale", default="",
                     help="override workload fields, e.g. 'prompts=1,group_sizes=2,T=2048' "
                          "(for profiling captures on a smaller case)")
