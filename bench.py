@@ -36,6 +36,13 @@ KERNEL_SRC = os.path.join(ROOT, "paper_2510_17158_gb300", "csrc", "gemm_tc.cu")
 GEMM_KERNELS = ("fwd_gemm_tc", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_tc")
 
 
+
+TILE_MODES = {0: "single CTA 128x256 (cta_group::1)",
+              1: "CTA pair 256x256 (cta_group::2)",
+              2: "2-CTA cluster, two 128x256 tiles sharing B by TMA multicast (cta_group::1)",
+              3: "4-CTA cluster, four 128x256 tiles sharing B by TMA multicast (cta_group::1)",
+              4: "2-CTA cluster, two 128x256 tiles sharing A by TMA multicast (cta_group::1)"}
+
 def peaks():
     try:
         p = json.load(open(PEAKS_PATH))
@@ -228,7 +235,9 @@ def run_gpu(args):
     dist_init(ws_n, "nccl")
     from paper_2510_17158_gb300 import grpo as G
     from paper_2510_17158_gb300.synthetic import WORKLOADS, lm_head_flops, make_batch_torch
-    G.grpo_set_cta_pair(bool(args.cta_pair))
+    G.grpo_set_tile_mode(args.tile_mode)
+    win = [int(x) for x in args.gemm_window.split(",")]
+    G.grpo_set_gemm_window(win[0], win[1])
     w = apply_scale(WORKLOADS[args.config], args.scale)
     w = w.scaled(seed=w.seed + 1000 * rank)        # each rank scores its own groups
     t_gen = time.time()
@@ -404,8 +413,9 @@ def run_gpu(args):
         "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
                    "d": d, "V": V, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
-                   "tiles": "CTA pair 256x256 (cta_group::2)" if args.cta_pair else
-                            "single CTA 128x256 (cta_group::1)",
+                   "tiles": TILE_MODES[args.tile_mode],
+                   "gemm_window": ("off" if win[0] == 0 else
+                                   f"{win[0]} k-blocks, lag {win[1]} checkpoints"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
                        b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
                    "parallelism": f"dp{ws_n} (independent groups per GPU)",
@@ -447,8 +457,11 @@ def main():
     ap.add_argument("--path", default="grpo", choices=["grpo", "sft", "grpo-exact-kl"],
                     help="grpo: the GRPO update (default); sft: the distillation loss step; "
                          "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
-    ap.add_argument("--cta-pair", type=int, default=0,
-                    help="tensor-core tiles: 0 = single CTAs (default), 1 = CTA pairs (cta_group::2)")
+    ap.add_argument("--tile-mode", type=int, default=0, choices=sorted(TILE_MODES),
+                    help="tensor-core tiles: " + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items()))
+    ap.add_argument("--gemm-window", default="0,0",
+                    help="GEMM progress window CHECK,LAG: producers stay within LAG checkpoints of "
+                         "CHECK k-blocks of the launch's average ('0,0' = off)")
     ap.add_argument("--graph", action="store_true",
                     help="capture one step in a CUDA graph and time its replays (per-kernel "
                          "timing and launch counts then come from the capture, not the replays)")

@@ -251,12 +251,42 @@ int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms);
  * such a call are undefined. Process-wide; not for production use. */
 int grpo_debug_inject_stall(int32_t on);
 
-/* Tensor-core tile shape of the four LM-head GEMMs, process-wide, for launches made afterwards:
- * on == 0 (default): one CTA per 128 x 256 tile (tcgen05 cta_group::1); on != 0: CTA pairs --
- * clusters of two CTAs on one TPC compute 256 x 256 tiles with cta_group::2, each CTA staging
- * half of B. Results agree within rounding. The pair mode does more work per clock, but on a
- * power-capped GB300 it draws more power per flop, so the single-CTA mode is the default. */
+/* Tensor-core tile mode of the LM-head GEMMs, process-wide, for launches made afterwards (the
+ * exact-KL GEMMs always use mode 0). Every mode computes the same 128-row output tiles with the
+ * same summation order inside a tile; modes 0, 2, 3 and 4 issue identical MMAs and give bitwise
+ * identical results, mode 1 (M = 256 MMAs) agrees within rounding.
+ *   GRPO_TILE_SINGLE     (0, default): one CTA per 128 x 256 tile (tcgen05 cta_group::1).
+ *   GRPO_TILE_CTA_PAIR   (1): clusters of two CTAs on one TPC compute 256 x 256 tiles with
+ *                        cta_group::2, each CTA staging half of B.
+ *   GRPO_TILE_MULTICAST  (2): clusters of two CTAs compute two 128 x 256 tiles that share a B
+ *                        tile; each CTA loads half of it and TMA multicast writes it to both.
+ *   GRPO_TILE_MULTICAST4 (3): the same with clusters of four CTAs, each loading a quarter of B.
+ *   GRPO_TILE_MULTICAST_A (4): clusters of two CTAs compute the tiles of one row tile and two
+ *                        adjacent column tiles, which share an A tile; each CTA loads half of
+ *                        its rows and TMA multicast writes them to both.
+ * Mode 0 is the default: on a power-capped GB300 it spends the least energy per flop of these
+ * (the step's throughput is bounded by the power cap, so energy per flop sets it).
+ * Returns GRPO_ERR_INVALID_ARG for any other mode. grpo_set_cta_pair(on) is mode 1 if on != 0,
+ * else mode 0; grpo_get_tile_mode returns the current mode. */
+enum {
+  GRPO_TILE_SINGLE = 0,
+  GRPO_TILE_CTA_PAIR = 1,
+  GRPO_TILE_MULTICAST = 2,
+  GRPO_TILE_MULTICAST4 = 3,
+  GRPO_TILE_MULTICAST_A = 4
+};
+int grpo_set_tile_mode(int32_t mode);
+int grpo_get_tile_mode(void);
 int grpo_set_cta_pair(int32_t on);
+
+/* Progress window of the tensor-core GEMMs, process-wide, for launches made afterwards. Every
+ * `check_kblocks` k-blocks of 64 the TMA producer of each CTA waits (at most 0.5 ms) until the
+ * CTAs of the launch are on average within `lag` such checkpoints of it, so that CTAs reading the
+ * same operand tiles read them close enough in time to hit L2 (long-K GEMMs otherwise drift apart
+ * and re-read their operands from HBM). Results do not depend on it. check_kblocks == 0 turns it
+ * off (the default: on a power-capped GB300 the waits cost more than the L2 hits gain). Returns GRPO_ERR_INVALID_ARG for negative values or for
+ * check_kblocks > 0 with lag == 0. */
+int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag);
 
 #ifdef __cplusplus
 }

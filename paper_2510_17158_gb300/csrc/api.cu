@@ -31,7 +31,8 @@ struct EventPair {
 std::mutex g_mu;
 std::atomic<int> g_timing{0};
 std::atomic<int> g_inject_stall{0};
-std::atomic<int> g_cta_pair{0};   // tensor-core tiles: 1 = CTA pairs (cta_group::2), 0 = single CTAs
+std::atomic<int> g_tile_mode{GRPO_TILE_SINGLE};  // tensor-core tile mode (GRPO_TILE_*)
+std::atomic<int> g_win_check{0}, g_win_lag{0};  // GEMM progress window (k-blocks, checkpoints)
 std::atomic<long long> g_launches[GRPO_K_COUNT];
 std::vector<EventPair> g_pending[GRPO_K_COUNT];
 double g_total_ms[GRPO_K_COUNT];
@@ -177,26 +178,6 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer
   return r == CUDA_SUCCESS;
 }
 
-int num_sms() {
-  int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-  return n;
-}
-
-// Persistent grid for `row_units` x `col_units` output tiles of 128 rows: one CTA per SM, or
-// one CTA pair per two SMs (then rows are paired and the grid is even).
-int gemm_grid(long long row_units, long long col_units, bool pair) {
-  const long long sms = num_sms();
-  if (sms <= 1) return pair ? 2 : 1;
-  if (!pair) {
-    const long long u = row_units * col_units;
-    return static_cast<int>(u < sms ? (u > 0 ? u : 1) : sms);
-  }
-  const long long pairs = ((row_units + 1) / 2) * col_units;
-  const long long cap = sms / 2;
-  return static_cast<int>(2 * (pairs < cap ? (pairs > 0 ? pairs : 1) : cap));
-}
 
 struct Views {
   WsHeader* hdr;
@@ -252,6 +233,7 @@ GemmArgs base_args(const Layout& L, const Views& v, int S, int T, int d, int V,
   a.rows_cap = L.rows_cap;
   a.num_strips = L.num_strips;
   a.inject_stall = g_inject_stall.load();
+  gemm_window_config(a);
   return a;
 }
 
@@ -359,17 +341,17 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   }
   if (!aligned16(H) || !aligned16(W)) return GRPO_ERR_INVALID_ARG;
   GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, valid_count, st));
-  const bool pair = g_cta_pair.load() != 0;
+  const int tm = gemm_role_tile_mode(ROLE_FWD);
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
-      !make_map(&mapW, W, d, V, d, pair ? kTileN / 2 : kTileN))
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+      !make_map(&mapW, W, d, V, d, gemm_b_box_rows(tm)))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
   a.partials = v.partials;
   a.zy = v.zy;
-  const int grid = gemm_grid(L.max_tiles, L.num_strips, pair);
+  const int grid = gemm_grid(L.max_tiles, L.num_strips, tm);
   GRPO_TRY(counted(GRPO_K_FWD_GEMM, st,
-                   [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st); }));
+                   [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, tm, st); }));
   return counted(GRPO_K_FWD_MERGE, st, [&] {
     return launch_fwd_merge(v.partials, L.rows_cap, L.num_strips, v.zy, v.pos_row, tokens,
                             mask, S, T, V, logp, lse, entropy, argmax, v.hdr, st);
@@ -478,14 +460,16 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
       return launch_gather_rows(H_ref, d, v.row_pos, v.hdr, L.rows_cap, v.hrp, st);
     }));
   }
-  const bool pair = g_cta_pair.load() != 0 && mode != 2;   // exact-KL roles: single-CTA tiles
+  // exact-KL roles: single-CTA tiles
+  const int tm = mode == 2 ? 0 : gemm_role_tile_mode(ROLE_DZ);
+  const int tm_dh = gemm_role_tile_mode(ROLE_DH), tm_dw = gemm_role_tile_mode(ROLE_DW);
   CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn, mapHrk, mapWrk;
   if (mode == 2 && (!make_map(&mapHrk, v.hrp, d, L.rows_cap, d, kTileRows) ||
                     !make_map(&mapWrk, W_ref, d, V, d, kTileN)))
     return GRPO_ERR_CUDA;
-  if (!make_map(&mapHk, v.hp, d, L.rows_cap, d, kTileRows) ||
-      !make_map(&mapWk, W, d, V, d, pair ? kTileN / 2 : kTileN) ||
-      !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
+  if (!make_map(&mapHk, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+      !make_map(&mapWk, W, d, V, d, gemm_b_box_rows(tm)) ||
+      !make_map(&mapDzK, dz, vc, L.rows_cap, vc, gemm_a_box_rows(tm_dh)) ||
       !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
       !make_map(&mapHmn, v.hp, d, L.rows_cap, d, 64))
     return GRPO_ERR_CUDA;
@@ -510,17 +494,18 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
     const long long vt = (a.vc_len + kTileN - 1) / kTileN;
     GRPO_TRY(counted(GRPO_K_BWD_DZ_GEMM, st, [&] {
       if (mode == 2)
-        return launch_gemm(ROLE_DZ_KL, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, false), false,
-                           st, &mapHrk, &mapWrk);
-      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, pair), pair, st);
+        return launch_gemm(ROLE_DZ_KL, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, 0), 0, st,
+                           &mapHrk, &mapWrk);
+      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, tm), tm, st);
     }));
     GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
-      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, d / kTileN, pair),
-                         pair, st);
+      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, d / kTileN, tm_dh),
+                         tm_dh, st);
     }));
     const long long vm = (a.vc_len + kTileRows - 1) / kTileRows;
     GRPO_TRY(counted(GRPO_K_BWD_DW_GEMM, st, [&] {
-      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, d / kTileN, pair), pair, st);
+      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, d / kTileN, tm_dw), tm_dw,
+                         st);
     }));
   }
   return counted(GRPO_K_DH_ZERO, st, [&] {
@@ -587,7 +572,7 @@ int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const voi
   a.partials2 = v.partials2;
   a.zy = v.zy;
   GRPO_TRY(counted(GRPO_K_FWD_GEMM, st, [&] {
-    return launch_gemm(ROLE_FWD_KL, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, false),
+    return launch_gemm(ROLE_FWD_KL, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, 0),
                        false, st, &mapHr, &mapWr);
   }));
   return counted(GRPO_K_FWD_MERGE, st, [&] {
@@ -627,18 +612,17 @@ int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);
   GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, v.counts, st));
-  const bool pair = g_cta_pair.load() != 0;
+  const int tm = gemm_role_tile_mode(ROLE_FWD);
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
-      !make_map(&mapW, W_shard, d, V_shard, d, pair ? kTileN / 2 : kTileN))
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+      !make_map(&mapW, W_shard, d, V_shard, d, gemm_b_box_rows(tm)))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V_shard, tokens, mask);
   a.v_offset = v_offset;
   a.partials = v.partials;
   a.zy = v.zy;
   GRPO_TRY(counted(GRPO_K_FWD_GEMM, st, [&] {
-    return launch_gemm(ROLE_FWD, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, pair), pair,
-                       st);
+    return launch_gemm(ROLE_FWD, mapH, mapW, a, gemm_grid(L.max_tiles, L.num_strips, tm), tm, st);
   }));
   return counted(GRPO_K_SHARD_STATS, st, [&] {
     return launch_shard_stats(v.partials, L.rows_cap, L.num_strips, v.zy, v.pos_row, tokens,
@@ -755,14 +739,37 @@ int grpo_debug_inject_stall(int32_t on) {
 }
 
 int grpo_set_cta_pair(int32_t on) {
-  g_cta_pair.store(on ? 1 : 0);
+  g_tile_mode.store(on ? 1 : 0);
+  return GRPO_OK;
+}
+
+int grpo_set_tile_mode(int32_t mode) {
+  if (mode < GRPO_TILE_SINGLE || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
+  g_tile_mode.store(mode);
+  return GRPO_OK;
+}
+
+int grpo_get_tile_mode(void) { return g_tile_mode.load(); }
+
+int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag) {
+  if (check_kblocks < 0 || lag < 0 || (check_kblocks > 0 && lag == 0)) return GRPO_ERR_INVALID_ARG;
+  g_win_check.store(check_kblocks);
+  g_win_lag.store(check_kblocks > 0 ? lag : 0);
   return GRPO_OK;
 }
 
 }  // extern "C"
 
 namespace grpo {
-bool gemm_pair_mode() { return g_cta_pair.load() != 0; }
+void gemm_window_config(GemmArgs& a) {
+  a.win_check = g_win_check.load();
+  a.win_lag = g_win_lag.load();
+}
+
+int gemm_role_tile_mode(int role) {
+  (void)role;   // one process-wide mode for the four GEMM roles
+  return g_tile_mode.load();
+}
 }  // namespace grpo
 
 extern "C" {

@@ -19,7 +19,11 @@ struct WsHeader {
   int32_t num_tiles;    // number of 128-token tiles of the current batch (tile list)
   int32_t pad0;
   long long total_valid;  // sum of valid counts
-  int32_t pad1[58];
+  // progress window of the tensor-core GEMMs: checkpoint arrivals of the running launch and the
+  // number of its CTAs that have left; the last CTA to leave resets both to 0
+  unsigned long long win_arrivals;
+  uint32_t win_exited;
+  int32_t pad1[55];
 };
 static_assert(sizeof(WsHeader) == 256, "header must be 256 bytes");
 
@@ -52,6 +56,13 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
+}
+
+// Relaxed load at GPU scope (a counter that other CTAs update with atomics).
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
 }
 
 // A kernel-internal wait gives up after this long and reports GRPO_ERR_TIMEOUT. The longest
@@ -297,6 +308,28 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst_smem, const CUtens
       "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst_smem),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+
+// TMA load whose box is written to the same shared-memory offset, and whose bytes are counted
+// on the mbarrier at the same offset, in every CTA of `cta_mask` within the cluster.
+__device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst_smem, const CUtensorMap* map,
+                                                      uint64_t* bar, int32_t x, int32_t y,
+                                                      uint16_t cta_mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst_smem),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(cta_mask)
+      : "memory");
+}
+
+// Arrive on `bar` (same CTA-local offset) in every CTA of `cta_mask` once all cta_group::1 MMAs
+// issued so far by this thread have completed.
+__device__ __forceinline__ void umma_commit_multicast(uint64_t* bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(cta_mask)
       : "memory");
 }
 

@@ -155,10 +155,10 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     if (rc != GRPO_OK) return rc;
     rc = ok_or_cuda(launch_gather_rows(H, d, row_pos, hdr, L.rows_cap, hp, st));
     if (rc != GRPO_OK) return rc;
-    const bool pair = gemm_pair_mode();
+    const int tm = gemm_role_tile_mode(ROLE_FWD);
     CUtensorMap mapH, mapW;
-    if (!bf16_map(&mapH, hp, d, static_cast<uint64_t>(L.rows_cap), kTileRows) ||
-        !bf16_map(&mapW, W, d, V, pair ? kTileN / 2 : kTileN))
+    if (!bf16_map(&mapH, hp, d, static_cast<uint64_t>(L.rows_cap), gemm_a_box_rows(tm)) ||
+        !bf16_map(&mapW, W, d, V, gemm_b_box_rows(tm)))
       return GRPO_ERR_CUDA;
     GemmArgs a;
     std::memset(&a, 0, sizeof(a));
@@ -174,20 +174,9 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     a.num_strips = L.num_strips;
     a.partials = partials;
     a.zy = zy;
-    int dev = 0, sms = 1;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-      return GRPO_ERR_CUDA;
-    int grid;
-    if (pair) {
-      const long long pairs = ((L.max_tiles + 1) / 2) * static_cast<long long>(L.num_strips);
-      const long long cap = sms / 2 > 0 ? sms / 2 : 1;
-      grid = static_cast<int>(2 * (pairs < cap ? (pairs > 0 ? pairs : 1) : cap));
-    } else {
-      const long long units = static_cast<long long>(L.max_tiles) * L.num_strips;
-      grid = static_cast<int>(units < sms ? (units > 0 ? units : 1) : sms);
-    }
-    rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, pair, st));
+    gemm_window_config(a);
+    const int grid = gemm_grid(L.max_tiles, L.num_strips, tm);
+    rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, tm, st));
     if (rc != GRPO_OK) return rc;
     rc = ok_or_cuda(launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, pos_row,
                                      tokens, mask, S, T, V, logp, lse, entropy, argmax, hdr, st));

@@ -18,6 +18,8 @@
 #include <cfloat>
 
 #include "common.cuh"
+#include <atomic>
+
 #include "internal.h"
 
 namespace grpo {
@@ -34,21 +36,37 @@ constexpr int NUM_THREADS = 192;
 #endif
 constexpr int GROUP_M = GRPO_GROUP_M;      // raster: row units sharing each column sweep
 
-// PAIR = false: one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128).
-// PAIR = true : a CTA pair (cluster of 2 on one TPC) computes a 256 x 256 tile with
-//               cta_group::2 (M = 256): each CTA stages its 128 rows of A and half (128 rows)
-//               of B, so per-SM operand traffic for B halves and the ring can be 6 deep.
-template <bool PAIR>
+// Tile modes (MODE template parameter):
+//   0 single CTA : one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128).
+//   1 CTA pair   : a cluster of 2 CTAs on one TPC computes a 256 x 256 tile with cta_group::2
+//                  (M = 256): each CTA stages its 128 rows of A and half (128 rows) of B, so the
+//                  per-SM operand traffic for B halves and the ring can be 6 deep.
+//   2, 3 B multicast: a cluster of CL = 2 (mode 2) or 4 (mode 3) CTAs computes CL 128 x 256
+//                  tiles of consecutive row tiles that share their B tile, with cta_group::1
+//                  MMAs; each CTA loads 1/CL of B and TMA multicast delivers it to all of them,
+//                  so per-CTA L2 -> SM traffic drops from 48 KB to 16 + 32/CL KB per k-block and
+//                  the CTAs of a cluster read B in lockstep.
+//   4 A multicast: a cluster of 2 CTAs computes the 128 x 256 tiles of one row tile and two
+//                  adjacent column tiles, which share their A tile; each CTA loads half of A's
+//                  rows and TMA multicast delivers them to both, so one read of an A tile from
+//                  HBM or L2 serves two column tiles.
+template <int MODE>
 struct Cfg {
-  static constexpr int STAGES = PAIR ? 6 : 4;
+  static constexpr int CL = MODE == 0 ? 1 : (MODE == 3 ? 4 : 2);      // CTAs per cluster
+  static constexpr bool MC_A = MODE == 4;                               // A shared by multicast
+  static constexpr bool MC_B = MODE == 2 || MODE == 3;                  // B shared by multicast
+  static constexpr uint16_t MASK = static_cast<uint16_t>((1u << CL) - 1u);
+  static constexpr int STAGES = MODE == 1 ? 6 : 4;
   static constexpr uint32_t A_STAGE = BM * BK * 2;                      // 16 KB
-  static constexpr uint32_t B_ROWS = PAIR ? BN / 2 : BN;                // B rows staged here
+  static constexpr uint32_t A_LOAD_ROWS = MC_A ? BM / CL : BM;          // A rows this CTA loads
+  static constexpr uint32_t B_ROWS = MODE == 1 ? BN / 2 : BN;           // B rows staged here
+  static constexpr uint32_t B_LOAD_ROWS =                               // B rows this CTA loads
+      MODE == 1 ? BN / 2 : (MC_B ? BN / CL : BN);
   static constexpr uint32_t B_STAGE = B_ROWS * BK * 2;                  // 16 or 32 KB
-  static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;               // bytes per CTA
+  static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;               // bytes landing per CTA
   static constexpr size_t SMEM = size_t(STAGES) * STAGE_TX + 1024 + 256;
 };
-constexpr size_t SMEM_BYTES = Cfg<false>::SMEM > Cfg<true>::SMEM ? Cfg<false>::SMEM
-                                                                  : Cfg<true>::SMEM;
+constexpr size_t SMEM_BYTES = Cfg<0>::SMEM > Cfg<1>::SMEM ? Cfg<0>::SMEM : Cfg<1>::SMEM;
 
 struct Dims {
   int num_m, num_n, num_kb;
@@ -77,13 +95,14 @@ __device__ __forceinline__ Dims role_dims(const GemmArgs& a, int num_tiles) {
   return d;
 }
 
-// Grouped raster: consecutive units walk GROUP_M row tiles before moving to the next column
+// Grouped raster: consecutive units walk `group` row units before moving to the next column
 // tile, so the CTAs resident at one time share a small set of A and B tiles in L2.
-__device__ __forceinline__ void decode_unit(int u, int num_m, int num_n, int& m, int& n) {
-  const int per_group = GROUP_M * num_n;
+__device__ __forceinline__ void decode_unit(int u, int num_m, int num_n, int group, int& m,
+                                            int& n) {
+  const int per_group = group * num_n;
   const int grp = u / per_group;
-  const int first_m = grp * GROUP_M;
-  const int gm = min(GROUP_M, num_m - first_m);
+  const int first_m = grp * group;
+  const int gm = min(group, num_m - first_m);
   const int within = u - grp * per_group;
   m = first_m + within % gm;
   n = within / gm;
@@ -105,68 +124,159 @@ __device__ __forceinline__ int acc_tiles_of_unit(const GemmArgs& a, int n) {
   return 1;
 }
 
-// Work layout shared by the three roles of a CTA. In PAIR mode a unit is a pair of M tiles
-// (2*mu for the leader CTA, 2*mu + 1 for its peer) and the pairs are strided over clusters.
-template <bool PAIR>
+// Work layout shared by the three roles of a CTA. In the cluster modes a unit is CL consecutive
+// M tiles with one N tile (CL*mu + rank for CTA `rank` of the cluster) and units are strided
+// over clusters.
+template <int MODE>
 struct Sched {
-  int rank;        // CTA rank in the pair (0 = leader, issues the MMAs); 0 without PAIR
+  int rank;        // CTA rank in the cluster (mode 1: 0 = leader, issues the MMAs); 0 in mode 0
+  int group;       // row units per raster group
   int first, step; // unit loop: u = first; u < num_units; u += step
-  int num_mu, num_units;
+  int num_mu, num_nu, num_units;
 
   __device__ __forceinline__ Sched(const Dims& dm) {
-    rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;
-    first = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
-    step = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
-    num_mu = PAIR ? (dm.num_m + 1) / 2 : dm.num_m;
-    num_units = num_mu * dm.num_n;
+    constexpr int CL = Cfg<MODE>::CL;
+    rank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+    first = static_cast<int>(blockIdx.x) / CL;
+    step = static_cast<int>(gridDim.x) / CL;
+    if (Cfg<MODE>::MC_A) {   // cluster spans column tiles
+      num_mu = dm.num_m;
+      num_nu = (dm.num_n + CL - 1) / CL;
+      group = GROUP_M;
+    } else {                 // cluster spans row tiles
+      num_mu = (dm.num_m + CL - 1) / CL;
+      num_nu = dm.num_n;
+      group = GROUP_M / CL > 0 ? GROUP_M / CL : 1;   // GROUP_M row tiles per raster group
+    }
+    num_units = num_mu * num_nu;
   }
-  // M tile of this CTA for unit row mu; `ok` false for the missing half of an odd tail pair
-  // (then `load` names a valid tile to stage, and nothing is stored).
-  __device__ __forceinline__ void m_of(int mu, int num_m, int& m, int& load, bool& ok) const {
-    m = PAIR ? 2 * mu + rank : mu;
-    ok = m < num_m;
-    load = ok ? m : (PAIR ? 2 * mu : mu);
+  // Unit u -> the row tile m and column unit n this CTA stages (always valid tiles), whether
+  // it stores its result (false for the CTAs of a cluster past the last row or, in mode 4,
+  // column tile, which only load their share of the shared operand) and the column unit n0
+  // whose accumulator count every CTA of the cluster uses: in mode 4 the CTAs of a cluster
+  // work on different column units, yet must issue the same k-blocks into the stages they
+  // share (a forward strip past the vocabulary's last tile reads zero-filled rows of W and
+  // adds nothing).
+  __device__ __forceinline__ void decode(int u, const Dims& dm, int& m, int& n, int& n0,
+                                         bool& ok) const {
+    constexpr int CL = Cfg<MODE>::CL;
+    int mu, nu;
+    decode_unit(u, num_mu, num_nu, group, mu, nu);
+    if (Cfg<MODE>::MC_A) {
+      m = mu;
+      n0 = CL * nu;
+      n = n0 + rank;
+      ok = n < dm.num_n;
+      if (!ok) n = n0;
+    } else {
+      m = CL * mu + rank;
+      n = n0 = nu;
+      ok = m < dm.num_m;
+      if (!ok) m = CL * mu;
+    }
   }
 };
 
 // ------------------------------------------------------------------------------------------
 // producer: one thread per CTA
 // ------------------------------------------------------------------------------------------
-template <int ROLE, bool PAIR>
+// Progress window. CTAs that read the same operand tile at the same k-block (a row tile of A
+// shared by the CTAs working on its other column tiles, or a column tile of B shared by the
+// CTAs on other row tiles) find it in L2 only if they read it within a few tens of microseconds
+// of one another: the L2 turns over that fast under these kernels' traffic. Over the thousands
+// of k-blocks of a long-K unit, CTAs otherwise drift apart by more than that. So every
+// `check` k-blocks the producer of each CTA counts itself in and waits until the CTAs of the
+// launch have, on average, reached `lag` checkpoints behind it. The slowest CTA never waits, so
+// the window cannot deadlock. It is a hint: a wait that runs past its bound switches the
+// window off for this CTA, and a CTA that leaves adds 2^40 so that no one waits for it.
+struct ProgressWindow {
+  unsigned long long* arrivals;
+  uint32_t* exited;
+  unsigned long long grid;
+  int check, lag;
+  bool on;
+  __device__ __forceinline__ ProgressWindow(const GemmArgs& a)
+      : arrivals(&a.hdr->win_arrivals), exited(&a.hdr->win_exited), grid(gridDim.x),
+        check(a.win_check), lag(a.win_lag), on(a.win_check > 0 && a.win_lag > 0) {}
+  __device__ __forceinline__ void at(long long kblocks_issued) {
+    if (!on || kblocks_issued == 0 || kblocks_issued % check != 0) return;
+    const long long c = kblocks_issued / check;
+    atomicAdd(arrivals, 1ull);
+    if (c < lag) return;
+    const unsigned long long target = grid * static_cast<unsigned long long>(c - lag + 1);
+    const uint64_t t0 = global_timer_ns();
+    while (ld_relaxed_u64(arrivals) < target) {
+      if (global_timer_ns() - t0 > 500000ull) {   // 0.5 ms: give up the window
+        on = false;
+        return;
+      }
+      __nanosleep(64);
+    }
+  }
+  __device__ __forceinline__ void leave() {
+    atomicAdd(arrivals, 1ull << 40);
+    __threadfence();
+    if (atomicAdd(exited, 1u) == static_cast<uint32_t>(grid - 1)) {   // last CTA: reset
+      atomicExch(arrivals, 0ull);
+      atomicExch(exited, 0u);
+    }
+  }
+};
+
+template <int ROLE, int MODE>
 __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
                              const CUtensorMap* mapA2, const CUtensorMap* mapB2, const GemmArgs& a,
-                             const Dims& dm, const Sched<PAIR>& sc, uint8_t* sA, uint8_t* sB,
+                             const Dims& dm, const Sched<MODE>& sc, uint8_t* sA, uint8_t* sB,
                              uint64_t* full, uint64_t* empty, volatile int* abort_flag) {
-  using C = Cfg<PAIR>;
-  const bool leader = sc.rank == 0;
+  using C = Cfg<MODE>;
+  // mode 1: only the leader's barriers count (both CTAs' bytes); modes 0, 2: every CTA's own
+  const bool leader = MODE != 1 || sc.rank == 0;
   const bool stall = (a.inject_stall != 0) && blockIdx.x == 0;   // CTA 0 is a leader
-  constexpr int B_BOXES = static_cast<int>(C::B_ROWS) / 64;      // MN-major B boxes per stage
-  const int b_col0 = PAIR ? sc.rank * static_cast<int>(C::B_ROWS) : 0;
+  constexpr int B_BOXES = static_cast<int>(C::B_LOAD_ROWS) / 64;  // MN-major B boxes loaded
+  constexpr int A_BOXES = static_cast<int>(C::A_LOAD_ROWS) / 64;  // MN-major A boxes loaded
+  const int b_col0 = (MODE == 1 || C::MC_B) ? sc.rank * static_cast<int>(C::B_LOAD_ROWS) : 0;
+  const int a_row0 = C::MC_A ? sc.rank * static_cast<int>(C::A_LOAD_ROWS) : 0;
+  // where this CTA's share of B (modes 2, 3) or A (mode 4) lands in every CTA's stage
+  const uint32_t b_off = C::MC_B ? sc.rank * C::B_LOAD_ROWS * BK * 2 : 0;
+  const uint32_t a_off = C::MC_A ? sc.rank * C::A_LOAD_ROWS * BK * 2 : 0;
   uint32_t stage = 0, phase = 0;
   long long issued = 0;
   bool ok = true;
+  ProgressWindow win(a);
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
-    int mu, n, m, m_load;
+    int m_load, n;
     bool m_ok;
-    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
-    sc.m_of(mu, dm.num_m, m, m_load, m_ok);
-    const int nacc = acc_tiles_of_unit<ROLE>(a, n);
+    int n0;
+    sc.decode(u, dm, m_load, n, n0, m_ok);
+    const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
     const int hrow = m_load * BM;   // first packed row of the tile (FWD / DZ / KL A operand)
     for (int t = 0; t < nacc && ok; ++t) {
       for (int kb = 0; kb < dm.num_kb; ++kb) {
+        win.at(issued);
         if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, a.hdr,
                                WHERE_GEMM_BASE + ROLE * 16 + 1)) {
           ok = false;
           break;
         }
-        const uint32_t dA = smem_u32(sA + stage * C::A_STAGE);
-        const uint32_t dB = smem_u32(sB + stage * C::B_STAGE);
-        // completion of both CTAs' copies is counted on the leader's barrier
-        const uint32_t bar = PAIR ? mapa_shared(smem_u32(&full[stage]), 0)
-                                  : smem_u32(&full[stage]);
-        auto load = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
-          if (PAIR) {
+        const uint32_t dA = smem_u32(sA + stage * C::A_STAGE) + a_off;
+        const uint32_t dB = smem_u32(sB + stage * C::B_STAGE) + b_off;
+        // mode 1: completion of both CTAs' copies is counted on the leader's barrier
+        const uint32_t bar = MODE == 1 ? mapa_shared(smem_u32(&full[stage]), 0)
+                                       : smem_u32(&full[stage]);
+        auto load_a = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
+          if (MODE == 1) {
             tma_load_2d_pair(dst, map, bar, x, y);
+          } else if (C::MC_A) {
+            tma_load_2d_multicast(dst, map, &full[stage], x, y, C::MASK);
+          } else {
+            tma_load_2d(dst, map, &full[stage], x, y);
+          }
+        };
+        auto load_b = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
+          if (MODE == 1) {
+            tma_load_2d_pair(dst, map, bar, x, y);
+          } else if (C::MC_B) {
+            tma_load_2d_multicast(dst, map, &full[stage], x, y, C::MASK);
           } else {
             tma_load_2d(dst, map, &full[stage], x, y);
           }
@@ -174,32 +284,32 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
         if (stall && issued == 0) {
           // test hook: leave stage 0 unfilled so that the MMA warp's bounded wait runs out
         } else {
-          if (leader) mbar_arrive_expect_tx(&full[stage], PAIR ? 2 * C::STAGE_TX : C::STAGE_TX);
+          if (leader) mbar_arrive_expect_tx(&full[stage], MODE == 1 ? 2 * C::STAGE_TX : C::STAGE_TX);
           if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
             const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
-            load(dA, mapA, kb * BK, hrow);
-            load(dB, mapB, kb * BK, vt * BN + b_col0);
+            load_a(dA, mapA, kb * BK, hrow + a_row0);
+            load_b(dB, mapB, kb * BK, vt * BN + b_col0);
           } else if (Dual<ROLE>::value) {
             // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
             const int nk = dm.num_kb / 2;
             const bool second = kb >= nk;
             const int kk = second ? kb - nk : kb;
             const int vt = (ROLE == ROLE_FWD_KL) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
-            load(dA, second ? mapA2 : mapA, kk * BK, hrow);
-            load(dB, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
+            load_a(dA, second ? mapA2 : mapA, kk * BK, hrow);
+            load_b(dB, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
           } else if (ROLE == ROLE_DH) {
-            load(dA, mapA, kb * BK, m_load * BM);
+            load_a(dA, mapA, kb * BK, m_load * BM + a_row0);
 #pragma unroll
             for (int j = 0; j < B_BOXES; ++j)
-              load(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kb * BK);
+              load_b(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kb * BK);
           } else {  // ROLE_DW
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j)
-              load(dA + j * BOX_MN, mapA, m_load * BM + j * 64, kb * BK);
+            for (int j = 0; j < A_BOXES; ++j)
+              load_a(dA + j * BOX_MN, mapA, m_load * BM + a_row0 + j * 64, kb * BK);
             const int row = kb * BK;    // K runs over packed rows
 #pragma unroll
             for (int j = 0; j < B_BOXES; ++j)
-              load(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, row);
+              load_b(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, row);
           }
         }
         ++issued;
@@ -210,10 +320,25 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
       }
     }
   }
+  if (ok && MODE != 0) {
+    // Cluster modes: the peer's MMAs release this CTA's stages by remote arrivals. Wait until
+    // every stage has been released for the last time, so that none of them lands after this
+    // CTA has left.
+    for (int i = 0; i < C::STAGES; ++i) {
+      if (!mbar_wait_bounded(&empty[stage], phase ^ 1u, abort_flag, a.hdr,
+                             WHERE_GEMM_BASE + ROLE * 16 + 1))
+        break;
+      if (++stage == C::STAGES) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  win.leave();
   if (!ok && leader) {
-    // Aborted: let the copies already in flight land before the CTA exits (bounded). In PAIR
-    // mode the leader's barriers also count the peer's copies; the peer waits for the leader
-    // at the final cluster barrier.
+    // Aborted: let the copies already in flight land before the CTA exits (bounded). In mode 1
+    // the leader's barriers also count the peer's copies; the peer waits for the leader at the
+    // final cluster barrier.
     const long long back = issued < C::STAGES ? issued : C::STAGES;
     for (long long i = 1; i <= back; ++i) {
       const long long it = issued - i;
@@ -226,14 +351,15 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
 }
 
 // ------------------------------------------------------------------------------------------
-// MMA issuer: one thread (of the leader CTA in PAIR mode)
+// MMA issuer: one thread (of the leader CTA in mode 1)
 // ------------------------------------------------------------------------------------------
-template <int ROLE, bool PAIR>
-__device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc, uint8_t* sA,
+template <int ROLE, int MODE>
+__device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc, uint8_t* sA,
                         uint8_t* sB, uint64_t* full, uint64_t* empty, uint64_t* accf,
                         uint64_t* acce, uint64_t* drain, uint32_t tmem_base,
                         volatile int* abort_flag) {
-  using C = Cfg<PAIR>;
+  using C = Cfg<MODE>;
+  constexpr bool PAIR = MODE == 1;
   if (PAIR && sc.rank != 0) return;
   constexpr bool A_MN = (ROLE == ROLE_DW);
   constexpr bool B_MN = (ROLE == ROLE_DH || ROLE == ROLE_DW);
@@ -241,9 +367,11 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
   uint32_t stage = 0, phase = 0, buf = 0, bphase = 0;
   bool ok = true;
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
-    int mu, n;
-    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
-    const int nacc = acc_tiles_of_unit<ROLE>(a, n);
+    int m_load, n;
+    bool m_ok;
+    int n0;
+    sc.decode(u, dm, m_load, n, n0, m_ok);
+    const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
     for (int t = 0; t < nacc && ok; ++t) {
       if (!mbar_wait_bounded(&acce[buf], bphase ^ 1u, abort_flag, a.hdr,
                              WHERE_GEMM_BASE + ROLE * 16 + 2)) {
@@ -278,9 +406,13 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc
             umma_bf16(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
           }
         }
-        // frees the smem stage (in both CTAs of a pair) once these MMAs have read it
+        // frees the smem stage once these MMAs have read it: mode 1 in both CTAs of the pair;
+        // modes 2, 3 tell every CTA of the cluster, because the next multicast into this stage
+        // writes all of them
         if (PAIR) {
           umma_commit_pair(&empty[stage], 0x3);
+        } else if (C::MC_A || C::MC_B) {
+          umma_commit_multicast(&empty[stage], C::MASK);
         } else {
           umma_commit(&empty[stage]);
         }
@@ -326,10 +458,11 @@ __device__ __forceinline__ bool epi_wait(uint64_t* bar, uint32_t parity, volatil
   return __all_sync(0xffffffffu, ok);
 }
 
-// Tells the MMA issuer that this warp has read accumulator `bar`'s buffer; in PAIR mode the
+// Tells the MMA issuer that this warp has read accumulator `bar`'s buffer; in mode 1 the
 // barrier lives in the leader CTA and counts the epilogue warps of both CTAs.
-template <bool PAIR>
+template <int MODE>
 __device__ __forceinline__ void epi_release(uint64_t* bar, int lane, int rank) {
+  constexpr bool PAIR = MODE == 1;
   tc_fence_before();
   __syncwarp();
   if (lane == 0) {
@@ -346,8 +479,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
-template <int ROLE, bool PAIR>
-__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR>& sc,
+template <int ROLE, int MODE>
+__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc,
                              uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
                              volatile int* abort_flag) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -357,10 +490,10 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
   const int32_t where = WHERE_GEMM_BASE + ROLE * 16 + 4;
   uint32_t buf = 0, bphase = 0;
   for (int u = sc.first; u < sc.num_units; u += sc.step) {
-    int mu, n, m, m_load;
-    bool m_ok;
-    decode_unit(u, sc.num_mu, dm.num_n, mu, n);
-    sc.m_of(mu, dm.num_m, m, m_load, m_ok);
+    int m_load, n;
+    bool m_ok;   // this CTA stores the tile (false: a cluster's CTA past the last tile)
+    int n0;
+    sc.decode(u, dm, m_load, n, n0, m_ok);
 
     if (ROLE == ROLE_FWD) {
       const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
@@ -371,7 +504,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       float rm = -INFINITY, rs = 0.f, ru = 0.f, zyv = 0.f;
       int ri = 0;
       bool found = false;
-      const int nacc = acc_tiles_of_unit<ROLE>(a, n);
+      const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
       for (int t = 0; t < nacc; ++t) {
         if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
         tc_fence_after();
@@ -423,12 +556,12 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
             found = true;
           }
         }
-        epi_release<PAIR>(&acce[buf], lane, sc.rank);
+        epi_release<MODE>(&acce[buf], lane, sc.rank);
         buf ^= 1u;
         if (buf == 0) bphase ^= 1u;
       }
       if (m_ok)
-        a.partials[static_cast<long long>(n) * a.rows_cap + static_cast<long long>(m) * BM + r] =
+        a.partials[static_cast<long long>(n) * a.rows_cap + static_cast<long long>(m_load) * BM + r] =
             make_float4(rm, rs, ru, __int_as_float(ri));
       if (found) a.zy[pos] = zyv;
 
@@ -442,7 +575,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
       float qm = -INFINITY, qs = 0.f;
       int ri = 0;
       bool found = false;
-      const int nacc = acc_tiles_of_unit<ROLE>(a, n);
+      const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
       for (int t = 0; t < nacc; ++t) {
         if (!epi_wait(&accf[0], bphase, abort_flag, a.hdr, where)) return;
         tc_fence_after();
@@ -508,12 +641,12 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
             found = true;
           }
         }
-        epi_release<PAIR>(&acce[0], lane, sc.rank);
+        epi_release<MODE>(&acce[0], lane, sc.rank);
         bphase ^= 1u;
       }
       if (m_ok) {
         const long long at = static_cast<long long>(n) * a.rows_cap +
-                             static_cast<long long>(m) * BM + r;
+                             static_cast<long long>(m_load) * BM + r;
         a.partials[at] = make_float4(rm, rs, ru, __int_as_float(ri));
         a.partials2[at] = make_float4(rc, qm, qs, 0.f);
       }
@@ -567,7 +700,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
         for (int j = 0; j < 4; ++j)
           dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
       }
-      epi_release<PAIR>(&acce[0], lane, sc.rank);
+      epi_release<MODE>(&acce[0], lane, sc.rank);
       bphase ^= 1u;
 
     } else if (ROLE == ROLE_DZ) {
@@ -608,7 +741,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
         for (int j = 0; j < 4; ++j)
           dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
       }
-      epi_release<PAIR>(&acce[buf], lane, sc.rank);
+      epi_release<MODE>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
 
@@ -623,7 +756,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
         if (!rv) continue;
-        float* acc_row = a.dH_acc + (static_cast<size_t>(m) * BM + r) * a.d + col;
+        float* acc_row = a.dH_acc + (static_cast<size_t>(m_load) * BM + r) * a.d + col;
         if (a.dh_mode == 2 || a.dh_mode == 3) {
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -654,12 +787,12 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
                                 pack_bf16x2(x[8 * j + 6], x[8 * j + 7]));
         }
       }
-      epi_release<PAIR>(&acce[buf], lane, sc.rank);
+      epi_release<MODE>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
 
     } else {  // ROLE_DW
-      const int vrow = m * BM + r;
+      const int vrow = m_load * BM + r;
       const bool rv = m_ok && vrow < a.vc_len;
       // No scored token at all (K = 0): no MMA ran, the accumulator holds nothing -> dW = 0.
       const bool empty_k = dm.num_kb == 0;
@@ -679,7 +812,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
         for (int j = 0; j < 8; ++j)
           dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
       }
-      epi_release<PAIR>(&acce[buf], lane, sc.rank);
+      epi_release<MODE>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
       if (buf == 0) bphase ^= 1u;
     }
@@ -689,11 +822,12 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<PAIR
 // ------------------------------------------------------------------------------------------
 // kernel body (both modes) and the two kernels
 // ------------------------------------------------------------------------------------------
-template <int ROLE, bool PAIR>
+template <int ROLE, int MODE>
 __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtensorMap* mapB,
                                           const CUtensorMap* mapA2, const CUtensorMap* mapB2,
                                           const GemmArgs& args) {
-  using C = Cfg<PAIR>;
+  using C = Cfg<MODE>;
+  constexpr bool PAIR = MODE == 1;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -712,7 +846,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], MODE >= 2 ? C::CL : 1);   // modes 2-4: every CTA's MMAs release
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
@@ -741,7 +875,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
     }
   }
   tc_fence_before();
-  if (PAIR) {
+  if (MODE != 0) {
     cluster_sync_all();  // barriers of both CTAs initialised before any cross-CTA traffic
   } else {
     __syncthreads();
@@ -749,23 +883,23 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const Dims dm = role_dims<ROLE>(args, args.hdr->num_tiles);
-  const Sched<PAIR> sc(dm);
+  const Sched<MODE> sc(dm);
 
   if (warp == 0) {
     if (lane == 0)
-      run_producer<ROLE, PAIR>(mapA, mapB, mapA2, mapB2, args, dm, sc, sA, sB, full, empty,
+      run_producer<ROLE, MODE>(mapA, mapB, mapA2, mapB2, args, dm, sc, sA, sB, full, empty,
                                abort_flag);
   } else if (warp == 1) {
     if (lane == 0)
-      run_mma<ROLE, PAIR>(args, dm, sc, sA, sB, full, empty, accf, acce, drain, tmem_base,
+      run_mma<ROLE, MODE>(args, dm, sc, sA, sB, full, empty, accf, acce, drain, tmem_base,
                           abort_flag);
   } else {
-    run_epilogue<ROLE, PAIR>(args, dm, sc, accf, acce, tmem_base, abort_flag);
+    run_epilogue<ROLE, MODE>(args, dm, sc, accf, acce, tmem_base, abort_flag);
   }
   __syncwarp();
   tc_fence_before();
-  if (PAIR) {
-    cluster_sync_all();  // no CTA leaves while its peer may still signal its barriers
+  if (MODE != 0) {
+    cluster_sync_all();  // no CTA leaves while its peer may still signal or write into it
   } else {
     __syncthreads();
   }
@@ -784,29 +918,81 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
             const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2,
             const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, false>(&mapA, &mapB, &mapA2, &mapB2, args);
+  gemm_body<ROLE, 0>(&mapA, &mapB, &mapA2, &mapB2, args);
 }
 
 template <int ROLE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_pair(const __grid_constant__ CUtensorMap mapA,
                  const __grid_constant__ CUtensorMap mapB, const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, true>(&mapA, &mapB, &mapA, &mapB, args);
+  gemm_body<ROLE, 1>(&mapA, &mapB, &mapA, &mapB, args);
+}
+
+template <int ROLE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_mc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+               const __grid_constant__ GemmArgs args) {
+  gemm_body<ROLE, 2>(&mapA, &mapB, &mapA, &mapB, args);
+}
+
+template <int ROLE>
+__global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_mc4(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                const __grid_constant__ GemmArgs args) {
+  gemm_body<ROLE, 3>(&mapA, &mapB, &mapA, &mapB, args);
+}
+
+template <int ROLE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_mca(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+                const __grid_constant__ GemmArgs args) {
+  gemm_body<ROLE, 4>(&mapA, &mapB, &mapA, &mapB, args);
 }
 
 template <int ROLE>
 cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const GemmArgs& args,
-                        int grid, bool pair, cudaStream_t st, const CUtensorMap& mapA2,
+                        int grid, int mode, cudaStream_t st, const CUtensorMap& mapA2,
                         const CUtensorMap& mapB2) {
-  if (pair && !Dual<ROLE>::value) {
-    const size_t smem = Cfg<true>::SMEM;
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair<ROLE>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    tc_gemm_pair<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
-  } else {
-    const size_t smem = Cfg<false>::SMEM;
+  if constexpr (!Dual<ROLE>::value) {       // exact-KL roles: single-CTA tiles only
+    if (mode == 1) {
+      const size_t smem = Cfg<1>::SMEM;
+      cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair<ROLE>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      tc_gemm_pair<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+      return cudaGetLastError();
+    }
+    if (mode == 2) {
+      const size_t smem = Cfg<2>::SMEM;
+      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mc<ROLE>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      tc_gemm_mc<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+      return cudaGetLastError();
+    }
+    if (mode == 3) {
+      const size_t smem = Cfg<3>::SMEM;
+      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mc4<ROLE>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      tc_gemm_mc4<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+      return cudaGetLastError();
+    }
+    if (mode == 4) {
+      const size_t smem = Cfg<4>::SMEM;
+      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mca<ROLE>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(smem));
+      if (e != cudaSuccess) return e;
+      tc_gemm_mca<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
+      return cudaGetLastError();
+    }
+  }
+  {
+    const size_t smem = Cfg<0>::SMEM;
     cudaError_t e = cudaFuncSetAttribute(tc_gemm<ROLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
@@ -819,22 +1005,82 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
 
 size_t gemm_smem_bytes() { return SMEM_BYTES; }
 
+int gemm_cluster_size(int tile_mode) { return tile_mode == 3 ? 4 : (tile_mode != 0 ? 2 : 1); }
+
+int gemm_b_box_rows(int tile_mode) {
+  return (tile_mode == 0 || tile_mode == 4) ? BN : BN / 2 / (tile_mode == 3 ? 2 : 1);
+}
+
+int gemm_a_box_rows(int tile_mode) { return tile_mode == 4 ? BM / 2 : BM; }
+
+namespace {
+template <typename Kernel>
+int query_active_clusters(Kernel kernel, size_t smem, int cl) {
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem)) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(cl), 1, 1);
+  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  int n = 0;   // the kernels fix their cluster shape at compile time: no attribute here
+  if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kernel), &cfg) !=
+      cudaSuccess) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_active_clusters[kMaxDevices][5];   // 0 = not queried yet
+}  // namespace
+
+int gemm_max_clusters(int tile_mode) {
+  const int cl = gemm_cluster_size(tile_mode);
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 1;
+  int cap = sms / cl > 0 ? sms / cl : 1;
+  if (cl == 1 || dev < 0 || dev >= kMaxDevices || tile_mode < 0 || tile_mode > 4) return cap;
+  int known = g_active_clusters[dev][tile_mode].load();
+  if (known == 0) {
+    int n = 0;
+    if (tile_mode == 1) n = query_active_clusters(tc_gemm_pair<ROLE_FWD>, Cfg<1>::SMEM, cl);
+    if (tile_mode == 2) n = query_active_clusters(tc_gemm_mc<ROLE_FWD>, Cfg<2>::SMEM, cl);
+    if (tile_mode == 3) n = query_active_clusters(tc_gemm_mc4<ROLE_FWD>, Cfg<3>::SMEM, cl);
+    if (tile_mode == 4) n = query_active_clusters(tc_gemm_mca<ROLE_FWD>, Cfg<4>::SMEM, cl);
+    known = n > 0 ? n : cap;   // a failed query falls back to one cluster per `cl` SMs
+    g_active_clusters[dev][tile_mode].store(known);
+  }
+  return known < cap ? known : cap;
+}
+
+int gemm_grid(long long row_units, long long col_units, int tile_mode) {
+  const long long cl = gemm_cluster_size(tile_mode);
+  const long long cap = gemm_max_clusters(tile_mode);
+  const long long units = tile_mode == 4 ? row_units * ((col_units + cl - 1) / cl)
+                                         : ((row_units + cl - 1) / cl) * col_units;
+  return static_cast<int>(cl * (units < cap ? (units > 0 ? units : 1) : cap));
+}
+
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, bool pair, cudaStream_t st,
+                        const GemmArgs& args, int grid, int mode, cudaStream_t st,
                         const CUtensorMap* mapA2, const CUtensorMap* mapB2) {
   const CUtensorMap& a2 = mapA2 ? *mapA2 : mapA;
   const CUtensorMap& b2 = mapB2 ? *mapB2 : mapB;
   switch (role) {
-    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, pair, st, a2, b2);
-    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, pair, st, a2, b2);
-    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, pair, st, a2, b2);
-    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, pair, st, a2, b2);
+    case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, mode, st, a2, b2);
+    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, mode, st, a2, b2);
+    case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, mode, st, a2, b2);
+    case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, mode, st, a2, b2);
     case ROLE_FWD_KL:
-      if (!mapA2 || !mapB2 || pair) return cudaErrorInvalidValue;
-      return launch_role<ROLE_FWD_KL>(mapA, mapB, args, grid, false, st, a2, b2);
+      if (!mapA2 || !mapB2 || mode != 0) return cudaErrorInvalidValue;
+      return launch_role<ROLE_FWD_KL>(mapA, mapB, args, grid, 0, st, a2, b2);
     case ROLE_DZ_KL:
-      if (!mapA2 || !mapB2 || pair) return cudaErrorInvalidValue;
-      return launch_role<ROLE_DZ_KL>(mapA, mapB, args, grid, false, st, a2, b2);
+      if (!mapA2 || !mapB2 || mode != 0) return cudaErrorInvalidValue;
+      return launch_role<ROLE_DZ_KL>(mapA, mapB, args, grid, 0, st, a2, b2);
     default: return cudaErrorInvalidValue;
   }
 }

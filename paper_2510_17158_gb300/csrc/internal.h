@@ -63,7 +63,13 @@ struct GemmArgs {
   const float* lse_ref;
   const float* kl;
   const float* c;
+  // progress window (0 = off): producers wait at every `win_check`-th k-block until the CTAs of
+  // the launch are on average within `win_lag` checkpoints of them (counters in hdr)
+  int win_check, win_lag;
 };
+
+// Fills the progress-window fields of `a` from the process-wide setting (grpo_set_gemm_window).
+void gemm_window_config(GemmArgs& a);
 
 // Launches (all asynchronous on `st`; return the cudaError_t of the launch).
 cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
@@ -126,15 +132,31 @@ cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
                           const uint8_t* mask, const float* lse, const float* g, int S, int T,
                           int d, int V, float* dW, cudaStream_t st);
 
-// Process-wide tensor-core tile mode chosen through grpo_set_cta_pair (true = CTA pairs).
-bool gemm_pair_mode();
+// Tensor-core tile mode (0 single CTA, 1 CTA pair with cta_group::2, 2 / 3 single-CTA MMAs
+// sharing B by TMA multicast in a 2- / 4-CTA cluster, 4 sharing A by TMA multicast in a 2-CTA
+// cluster) that GEMM role `role` (ROLE_*) runs in,
+// (the process-wide mode chosen through grpo_set_tile_mode).
+int gemm_role_tile_mode(int role);
 
 // tcgen05 GEMM launches. `grid` = persistent CTAs.
 size_t gemm_smem_bytes();
-// pair = true: CTA-pair kernels (clusters of 2, cta_group::2); `grid` must then be even.
+// CTAs per cluster of a tile mode (1, 2 or 4) and the rows of the K-major B box each CTA loads.
+int gemm_cluster_size(int tile_mode);
+int gemm_b_box_rows(int tile_mode);
+// Rows of the K-major A box each CTA loads (64 in mode 4, where two CTAs share A; else 128).
+int gemm_a_box_rows(int tile_mode);
+// Clusters of a tile mode that can be resident at once (cudaOccupancyMaxActiveClusters, cached
+// per device), at most one per `cluster size` SMs.
+int gemm_max_clusters(int tile_mode);
+// Persistent grid for `row_units` x `col_units` output tiles of 128 rows: one CTA per SM, or in
+// the cluster modes as many clusters as can be resident, each taking `cluster size`
+// consecutive row tiles per unit; never more CTAs than units need.
+int gemm_grid(long long row_units, long long col_units, int tile_mode);
+// tile_mode 1, 2, 3: cluster kernels; `grid` must be a multiple of the cluster size and the
+// K-major B map's box gemm_b_box_rows(tile_mode) rows (each CTA loads its share of B).
 // mapA2 / mapB2 (H_ref, W_ref) are read by the KL roles only (single-CTA tiles).
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
-                        const GemmArgs& args, int grid, bool pair, cudaStream_t st,
+                        const GemmArgs& args, int grid, int tile_mode, cudaStream_t st,
                         const CUtensorMap* mapA2 = nullptr, const CUtensorMap* mapB2 = nullptr);
 
 }  // namespace grpo

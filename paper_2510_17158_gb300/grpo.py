@@ -61,6 +61,9 @@ def _declare(lib):
         "grpo_timing_read": (ctypes.c_int, [_i32, ctypes.POINTER(_i64), ctypes.POINTER(_f64)]),
         "grpo_debug_inject_stall": (ctypes.c_int, [_i32]),
         "grpo_set_cta_pair": (ctypes.c_int, [_i32]),
+        "grpo_set_tile_mode": (ctypes.c_int, [_i32]),
+        "grpo_get_tile_mode": (ctypes.c_int, []),
+        "grpo_set_gemm_window": (ctypes.c_int, [_i32, _i32]),
         "grpo_sft_loss_bwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                              _p, _p, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
         "grpo_rewards": (ctypes.c_int, [_p, _p, _p, _p, _p, _i32, _f32, _p, _p]),
@@ -469,6 +472,25 @@ def grpo_debug_inject_stall(on: bool):
 
 def grpo_set_cta_pair(on: bool):
     _check(_lib().grpo_set_cta_pair(1 if on else 0), "grpo_set_cta_pair")
+
+
+TILE_SINGLE, TILE_CTA_PAIR, TILE_MULTICAST, TILE_MULTICAST4, TILE_MULTICAST_A = 0, 1, 2, 3, 4
+
+
+def grpo_set_tile_mode(mode: int):
+    """0 single-CTA tiles (default), 1 CTA pairs (cta_group::2), 2 / 3 B tile shared by TMA
+    multicast in clusters of 2 / 4 CTAs, 4 A tile shared by TMA multicast in 2-CTA clusters."""
+    _check(_lib().grpo_set_tile_mode(int(mode)), "grpo_set_tile_mode")
+
+
+def grpo_get_tile_mode() -> int:
+    return int(_lib().grpo_get_tile_mode())
+
+
+def grpo_set_gemm_window(check_kblocks: int, lag: int):
+    """GEMM progress window: producers stay within `lag` checkpoints of `check_kblocks` k-blocks
+    of the launch's average (0 turns it off, the default)."""
+    _check(_lib().grpo_set_gemm_window(int(check_kblocks), int(lag)), "grpo_set_gemm_window")
 
 
 def timing_table() -> dict:

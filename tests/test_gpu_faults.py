@@ -72,14 +72,18 @@ def test_bad_group_offsets_set_status():
     assert np.isfinite(a.cpu().numpy()).all()
 
 
-def test_stalled_pipeline_times_out_in_cta_pair_mode():
-    """The same injected stall with CTA-pair tiles: the leader's MMA wait runs out, both CTAs of
-    every pair leave through their bounded waits and the final cluster barrier, and the next
-    call is correct."""
+@pytest.mark.parametrize("mode", [1, 2, 3, 4],
+                         ids=["cta_pair", "multicast2", "multicast4", "multicast_a"])
+def test_stalled_pipeline_times_out_in_cluster_tile_modes(mode):
+    """The same injected stall with 2-CTA clusters. Mode 1 (CTA pairs): the leader's MMA wait
+    runs out. Modes 2-4 (B or A multicast): CTA 0 loads neither its own operand nor its share of
+    the shared one, so the MMA waits of every CTA in its cluster run out. Every CTA leaves through its bounded waits and the final
+    cluster barrier, and the next call is correct."""
     b, (H, W, tok, mask) = _small()
     S, T, d = H.shape
     ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
-    G.grpo_set_cta_pair(True)
+    prev = G.grpo_get_tile_mode()
+    G.grpo_set_tile_mode(mode)
     try:
         good = {k: v.clone() for k, v in G.grpo_score_fwd(H, W, tok, mask, ws).items()}
         assert G.grpo_last_device_error(ws)[0] == 0
@@ -96,4 +100,4 @@ def test_stalled_pipeline_times_out_in_cta_pair_mode():
         for k in ("logp", "lse", "entropy", "argmax"):
             assert torch.equal(again[k], good[k]), k
     finally:
-        G.grpo_set_cta_pair(False)
+        G.grpo_set_tile_mode(prev)

@@ -114,22 +114,47 @@ def test_deterministic_bitwise():
     assert g1["loss"] == g2["loss"]
 
 
-def test_pair_tiles_match_oracle_and_single_cta_tiles():
-    """The CTA-pair tile mode (M = 256, cta_group::2) and the default 1-CTA mode (M = 128,
-    cta_group::1) both meet the parity bar and agree with each other."""
+@pytest.mark.parametrize("name", ["d4096_v152k", "d2048_v32k"])
+def test_tile_modes_match_oracle_and_single_cta_tiles(name):
+    """Every tile mode meets the parity bar: 0 (the default, one CTA per 128 x 256 tile), 1 (CTA
+    pairs, M = 256, cta_group::2), 2 / 3 (two / four 1-CTA tiles sharing their B tile by TMA
+    multicast) and 4 (two 1-CTA tiles of adjacent column tiles sharing their A tile). Modes 2, 3
+    and 4 issue the same MMAs in the same order as mode 0, so their outputs are bitwise equal to
+    mode 0's; mode 1 agrees within rounding. The d2048 case packs into 85 row tiles (85 = 2*42 + 1 = 4*21 + 1), so CTAs of the
+    last cluster have no tile of their own and only load their share of B for the others."""
     from paper_2510_17158_gb300 import grpo as G
-    b = _batch("d4096_v152k")
+    b = _batch(name)
     old, ref = oracle_inputs(b)
-    G.grpo_set_cta_pair(True)
-    try:
-        g1 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
-    finally:
-        G.grpo_set_cta_pair(False)
-    g2 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
     o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
-    print(compare(b, g1, o), compare(b, g2, o))
-    for k in ("logp", "lse", "entropy"):
-        assert float((g1[k] - g2[k]).abs().max()) <= 1e-4
+    prev = G.grpo_get_tile_mode()
+    assert prev == G.TILE_SINGLE                     # the library's default
+    try:
+        G.grpo_set_tile_mode(G.TILE_SINGLE)
+        g0 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+        print("mode 0", compare(b, g0, o))
+        for mode in (G.TILE_CTA_PAIR, G.TILE_MULTICAST, G.TILE_MULTICAST4, G.TILE_MULTICAST_A):
+            G.grpo_set_tile_mode(mode)
+            assert G.grpo_get_tile_mode() == mode
+            g = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+            print("mode", mode, compare(b, g, o))
+            if mode == G.TILE_CTA_PAIR:
+                for k in ("logp", "lse", "entropy"):
+                    assert float((g[k] - g0[k]).abs().max()) <= 1e-4, k
+            else:
+                for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
+                    assert torch.equal(g[k], g0[k]), (mode, k)
+                assert g["loss"] == g0["loss"]
+    finally:
+        G.grpo_set_tile_mode(prev)
+
+
+def test_tile_mode_rejects_unknown_modes():
+    from paper_2510_17158_gb300 import grpo as G
+    prev = G.grpo_get_tile_mode()
+    for bad in (-1, 5):
+        with pytest.raises(G.GrpoError):
+            G.grpo_set_tile_mode(bad)
+    assert G.grpo_get_tile_mode() == prev
 
 
 def test_chunked_backward_full_vocabulary_partial_last_chunk():
@@ -145,3 +170,35 @@ def test_chunked_backward_full_vocabulary_partial_last_chunk():
     g = run_gpu(b, old, ref, 0.2, 0.2, 0.04, vocab_chunk=40960)
     o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
     print(compare(b, g, o))
+
+
+def test_progress_window_changes_nothing_and_resets_its_counters():
+    """The GEMM progress window only delays TMA issue: outputs with it off (the default), at 16
+    k-blocks with lag 4 and at a tight setting (1 k-block, lag 1, so that the producers wait at
+    every k-block) are bitwise equal, and the last CTA of every launch resets the window's
+    counters in the workspace header (arrivals at byte 24, CTAs left at byte 32) to 0."""
+    from paper_2510_17158_gb300 import grpo as G
+    b = _batch("d4096_v152k")
+    old, ref = oracle_inputs(b)
+    outs = []
+    try:
+        for check, lag in ((0, 0), (16, 4), (1, 1)):
+            G.grpo_set_gemm_window(check, lag)
+            outs.append(run_gpu(b, old, ref, 0.2, 0.2, 0.04))
+            dev = torch.device("cuda")
+            H, W = b.H.to(dev), b.W.to(dev)
+            S, T, d = H.shape
+            ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
+            G.grpo_score_fwd(H, W, b.tokens.to(dev), b.mask.to(dev), ws)
+            torch.cuda.synchronize()
+            hdr = ws.buf[:64].cpu().numpy()
+            assert int(hdr[24:32].view(np.uint64)[0]) == 0
+            assert int(hdr[32:36].view(np.uint32)[0]) == 0
+    finally:
+        G.grpo_set_gemm_window(0, 0)
+    for g in outs[1:]:
+        for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
+            assert torch.equal(g[k], outs[0][k]), k
+        assert g["loss"] == outs[0]["loss"]
+    with pytest.raises(G.GrpoError):
+        G.grpo_set_gemm_window(16, 0)
