@@ -250,6 +250,35 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
     sc.decode(u, dm, m_load, n, n0, m_ok);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
     const int hrow = m_load * BM;   // first packed row of the tile (FWD / DZ / KL A operand)
+    // The boxes of k-block kbi of accumulator tile ti: fa / fb(smem offset, map, x, y) for each
+    // box of A / B this CTA loads.
+    auto boxes = [&](int ti, int kbi, auto&& fa, auto&& fb) {
+      if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
+        const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + ti : a.vc0 / BN + n;
+        fa(0u, mapA, kbi * BK, hrow + a_row0);
+        fb(0u, mapB, kbi * BK, vt * BN + b_col0);
+      } else if (Dual<ROLE>::value) {
+        // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
+        const int nk = dm.num_kb / 2;
+        const bool second = kbi >= nk;
+        const int kk = second ? kbi - nk : kbi;
+        const int vt = (ROLE == ROLE_FWD_KL) ? n * kFwdTilesPerStrip + ti : a.vc0 / BN + n;
+        fa(0u, second ? mapA2 : mapA, kk * BK, hrow);
+        fb(0u, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
+      } else if (ROLE == ROLE_DH) {
+        fa(0u, mapA, kbi * BK, m_load * BM + a_row0);
+#pragma unroll
+        for (int j = 0; j < B_BOXES; ++j)
+          fb(j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kbi * BK);
+      } else {  // ROLE_DW: K runs over packed rows
+#pragma unroll
+        for (int j = 0; j < A_BOXES; ++j)
+          fa(j * BOX_MN, mapA, m_load * BM + a_row0 + j * 64, kbi * BK);
+#pragma unroll
+        for (int j = 0; j < B_BOXES; ++j)
+          fb(j * BOX_MN, mapB, n * BN + b_col0 + j * 64, kbi * BK);
+      }
+    };
     for (int t = 0; t < nacc && ok; ++t) {
       for (int kb = 0; kb < dm.num_kb; ++kb) {
         win.at(issued);
@@ -263,54 +292,29 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
         // mode 1: completion of both CTAs' copies is counted on the leader's barrier
         const uint32_t bar = MODE == 1 ? mapa_shared(smem_u32(&full[stage]), 0)
                                        : smem_u32(&full[stage]);
-        auto load_a = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
+        auto load_a = [&](uint32_t off, const CUtensorMap* map, int x, int y) {
           if (MODE == 1) {
-            tma_load_2d_pair(dst, map, bar, x, y);
+            tma_load_2d_pair(dA + off, map, bar, x, y);
           } else if (C::MC_A) {
-            tma_load_2d_multicast(dst, map, &full[stage], x, y, C::MASK);
+            tma_load_2d_multicast(dA + off, map, &full[stage], x, y, C::MASK);
           } else {
-            tma_load_2d(dst, map, &full[stage], x, y);
+            tma_load_2d(dA + off, map, &full[stage], x, y);
           }
         };
-        auto load_b = [&](uint32_t dst, const CUtensorMap* map, int x, int y) {
+        auto load_b = [&](uint32_t off, const CUtensorMap* map, int x, int y) {
           if (MODE == 1) {
-            tma_load_2d_pair(dst, map, bar, x, y);
+            tma_load_2d_pair(dB + off, map, bar, x, y);
           } else if (C::MC_B) {
-            tma_load_2d_multicast(dst, map, &full[stage], x, y, C::MASK);
+            tma_load_2d_multicast(dB + off, map, &full[stage], x, y, C::MASK);
           } else {
-            tma_load_2d(dst, map, &full[stage], x, y);
+            tma_load_2d(dB + off, map, &full[stage], x, y);
           }
         };
         if (stall && issued == 0) {
           // test hook: leave stage 0 unfilled so that the MMA warp's bounded wait runs out
         } else {
           if (leader) mbar_arrive_expect_tx(&full[stage], MODE == 1 ? 2 * C::STAGE_TX : C::STAGE_TX);
-          if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
-            const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
-            load_a(dA, mapA, kb * BK, hrow + a_row0);
-            load_b(dB, mapB, kb * BK, vt * BN + b_col0);
-          } else if (Dual<ROLE>::value) {
-            // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
-            const int nk = dm.num_kb / 2;
-            const bool second = kb >= nk;
-            const int kk = second ? kb - nk : kb;
-            const int vt = (ROLE == ROLE_FWD_KL) ? n * kFwdTilesPerStrip + t : a.vc0 / BN + n;
-            load_a(dA, second ? mapA2 : mapA, kk * BK, hrow);
-            load_b(dB, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
-          } else if (ROLE == ROLE_DH) {
-            load_a(dA, mapA, kb * BK, m_load * BM + a_row0);
-#pragma unroll
-            for (int j = 0; j < B_BOXES; ++j)
-              load_b(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kb * BK);
-          } else {  // ROLE_DW
-#pragma unroll
-            for (int j = 0; j < A_BOXES; ++j)
-              load_a(dA + j * BOX_MN, mapA, m_load * BM + a_row0 + j * 64, kb * BK);
-            const int row = kb * BK;    // K runs over packed rows
-#pragma unroll
-            for (int j = 0; j < B_BOXES; ++j)
-              load_b(dB + j * BOX_MN, mapB, n * BN + b_col0 + j * 64, row);
-          }
+          boxes(t, kb, load_a, load_b);
         }
         ++issued;
         if (++stage == C::STAGES) {
