@@ -144,7 +144,13 @@ class ClockSampler:
 
 
 def kernel_source_sha() -> str:
-    return hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()[:16]
+    """Hash of the GEMM kernel's code with comments and blank lines removed (a comment edit does
+    not invalidate a committed traffic measurement; any code change does)."""
+    txt = open(KERNEL_SRC).read()
+    txt = re.sub(r"//[^\n]*", "", txt)
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    txt = "\n".join(line.strip() for line in txt.splitlines() if line.strip())
+    return hashlib.sha256(txt.encode()).hexdigest()[:16]
 
 
 def ncu_traffic(kernel: str, workload: str):

@@ -13,8 +13,9 @@
 // (bf16 in, f32 accumulate in tensor memory), warps 2-5 read the accumulator back with
 // tcgen05.ld (one TMEM lane = one output row per thread) and run the role's epilogue. Two
 // 256-column accumulators in TMEM let the epilogue of one tile overlap the MMAs of the next.
-// Two modes: one CTA per 128 x 256 tile (cta_group::1), or a CTA pair per 256 x 256 tile
-// (cta_group::2, see Cfg). Every wait is bounded (see mbar_wait_bounded).
+// Tile modes (see Cfg): one CTA per 128 x 256 tile (cta_group::1, the default), a CTA pair per
+// 256 x 256 tile (cta_group::2), or 2- / 4-CTA clusters whose CTAs share one operand tile by
+// TMA multicast. Every wait is bounded (see mbar_wait_bounded).
 #include <cfloat>
 
 #include "common.cuh"
@@ -824,7 +825,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
 }
 
 // ------------------------------------------------------------------------------------------
-// kernel body (both modes) and the two kernels
+// kernel body (every tile mode) and one kernel per mode
 // ------------------------------------------------------------------------------------------
 template <int ROLE, int MODE>
 __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtensorMap* mapB,
