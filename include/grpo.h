@@ -4,7 +4,7 @@
  * One GRPO update (arxiv 2510.17158, Alg. 1) scores K sampled completions per prompt, normalises
  * their rewards within the group, and takes a gradient step on
  *     L = E_{x~pi}[ -w(x) log pi(x|c) ] + beta KL(pi || pi_ref)                  (Eq. 1)
- * using the clipped-ratio surrogate that Sec. 6.1 keeps from "traditional GRPO". This library
+ * using the clipped-ratio surrogate of standard GRPO, which Sec. 6.1 keeps. This library
  * computes the data-parallel core of that step for the LM head: logits z = W h per token over
  * the whole vocabulary (never written to memory), log-softmax at the sampled token, entropy and
  * argmax, group advantages, the per-token surrogate + KL loss, and dL/dH, dL/dW.
@@ -67,7 +67,8 @@ size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t 
 /* Clears the workspace's status word. Call once after allocating a workspace. */
 int grpo_workspace_init(void* workspace, size_t workspace_bytes, grpo_stream_t stream);
 
-/* Group-relative advantages (Eq. 1's w(x); Sec. 2.1 and Alg. 1 "normalize within each group").
+/* Group-relative advantages (Eq. 1's w(x): rewards normalised within each group, Sec. 2.1 and
+ * Alg. 1).
  *   rewards        [num_seqs] f32
  *   group_offsets  [num_groups+1] int32, device; must rise from 0 to num_seqs (else the status
  *                  word gets GRPO_ERR_GROUPS and the affected advantages are NaN)

@@ -6,11 +6,10 @@ imports nothing from the package: callers hand it plain numpy arrays.
 
 What it computes (arxiv 2510.17158):
 
-* Eq. 1 (Sec. 2.1, "Fine-tuning LMs with RL") is the GRPO objective
+* Eq. 1 (Sec. 2.1) is the GRPO objective
   ``L = E_{x~pi}[-w(x) log pi(x|c)] + beta KL(pi || pi_ref)``, where ``w(x)`` is the reward of
-  ``x`` normalised within its group of K completions (Sec. 2.1; Alg. 1, "normalize within each
-  group").
-* Sec. 6.1 ("GRPO Adaptations") keeps "the traditional GRPO policy" of DeepSeekMath, i.e. the
+  ``x`` normalised within its group of K completions (Sec. 2.1; Alg. 1).
+* Sec. 6.1 keeps the standard GRPO policy update of DeepSeekMath, i.e. the
   per-token probability ratio with a clipped surrogate; Alg. 1 computes the KL to a frozen
   reference and takes a gradient step on L.
 * ``log pi(x|c)`` is the sum over the completion's sampled tokens of the log-softmax of the
@@ -30,7 +29,7 @@ Readings of points the paper leaves open (each one is a documented choice):
   inclusive boundaries: active iff (A >= 0 and rho <= 1+eps_hi) or (A < 0 and rho >= 1-eps_lo);
 * argmax ties go to the lowest vocabulary index; entropy is in nats;
 * distillation (Sec. 6.2) is token cross-entropy with the same aggregation choices;
-* the performance reward's "correct but slower" is t > t_base.
+* the performance reward's branch for a correct but slower kernel is t > t_base.
 
 Every input is converted exactly to float64 (bf16 and fp32 values are exactly representable).
 """
@@ -55,8 +54,8 @@ def valid_counts(mask):
 
 
 def group_advantages(rewards, group_offsets, std_mode="unbiased", std_eps=1e-4):
-    """w(x_k) of Eq. 1: the reward of completion k normalised within its group (Sec. 2.1;
-    Alg. 1, "normalize within each group to get advantages").
+    """w(x_k) of Eq. 1: the reward of completion k normalised within its group, which Alg. 1
+    turns into the advantages (Sec. 2.1; Alg. 1).
 
     ``group_offsets[g] .. group_offsets[g+1]`` are the completions of prompt g (contiguous).
     """

@@ -16,7 +16,7 @@ namespace grpo {
 struct WsHeader {
   int32_t status;       // first device-side error (grpo_status), 0 = none
   int32_t where;        // code of the kernel/wait that recorded it
-  int32_t num_tiles;    // number of 128-token tiles of the current batch (tile list)
+  int32_t num_tiles;    // number of 128-row tiles of packed scored tokens of the current batch
   int32_t pad0;
   long long total_valid;  // sum of valid counts
   // progress window of the tensor-core GEMMs: checkpoint arrivals of the running launch and the

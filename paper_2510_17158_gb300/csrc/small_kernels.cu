@@ -1,6 +1,6 @@
 // Reduction and bookkeeping kernels of the GRPO path, plus the f32 CUDA-core path for small
-// problems: valid-token counts and the token-tile list, group-relative advantages (Eq. 1's
-// w(x), Alg. 1 "normalize within each group"), the merge of per-strip softmax statistics into
+// problems: valid-token counts and the packed token rows, group-relative advantages (Eq. 1's
+// w(x): rewards normalised within each group, Alg. 1), the merge of per-strip softmax statistics into
 // logp / lse / entropy / argmax, and the per-token clipped surrogate + KL loss with its
 // coefficient g_t = dL/dlogp_t (Sec. 6.1, Eq. 1). All reductions use a fixed order, so results
 // are bitwise reproducible run to run.
