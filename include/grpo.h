@@ -83,7 +83,7 @@ int group_advantages(const float* rewards, const int32_t* group_offsets, int32_t
  * chip (the [tokens x V] logits never reach memory) to
  *   lse_t = log sum_v exp(z_tv), logp_t = z_t[y_t] - lse_t, entropy_t = lse_t - sum_v p_tv z_tv
  *   (nats), argmax_t = lowest v with the largest z_tv; valid_count_i = #scored tokens of seq i.
- * dtype GRPO_BF16: bf16 H, W, tensor-core products with f32 accumulation (d % 256 == 0).
+ * dtype GRPO_BF16: bf16 H, W, tensor-core products with f32 accumulation (d % 64 == 0).
  * dtype GRPO_F32 : f32 H, W, f32 CUDA-core arithmetic (small problems, d <= 4096).
  * Outputs: logp, lse, entropy f32 [S,T]; argmax int32 [S,T]; valid_count int32 [S]. */
 int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* tokens,

@@ -133,7 +133,7 @@ bool shape_ok(int S, int T, int d, int V) {
 }
 
 int check_dtype_shape(int dtype, int d) {
-  if (dtype == GRPO_BF16) return (d % kTileN == 0) ? GRPO_OK : GRPO_ERR_UNSUPPORTED;
+  if (dtype == GRPO_BF16) return (d % 64 == 0) ? GRPO_OK : GRPO_ERR_UNSUPPORTED;
   if (dtype == GRPO_F32) return (d <= 4096) ? GRPO_OK : GRPO_ERR_UNSUPPORTED;
   return GRPO_ERR_INVALID_ARG;
 }
@@ -487,6 +487,7 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   a.dH = static_cast<__nv_bfloat16*>(dH);
   a.dH_acc = dH_acc;
   a.dW = dW;
+  const long long dtiles = (d + kTileN - 1) / kTileN;   // output column tiles of dH and dW
   for (int c = 0; c < nchunks; ++c) {
     a.vc0 = c * vc;
     a.vc_len = (V - a.vc0) < vc ? (V - a.vc0) : vc;
@@ -499,12 +500,12 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
       return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, tm), tm, st);
     }));
     GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
-      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, d / kTileN, tm_dh),
+      return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, dtiles, tm_dh),
                          tm_dh, st);
     }));
     const long long vm = (a.vc_len + kTileRows - 1) / kTileRows;
     GRPO_TRY(counted(GRPO_K_BWD_DW_GEMM, st, [&] {
-      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, d / kTileN, tm_dw), tm_dw,
+      return launch_gemm(ROLE_DW, mapDzMn, mapHmn, a, gemm_grid(vm, dtiles, tm_dw), tm_dw,
                          st);
     }));
   }

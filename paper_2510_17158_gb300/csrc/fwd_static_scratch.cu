@@ -116,7 +116,7 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
       V >= (1 << 30))
     return GRPO_ERR_INVALID_ARG;
   if (dtype == GRPO_BF16) {
-    if (d % kTileN != 0) return GRPO_ERR_UNSUPPORTED;
+    if (d % 64 != 0) return GRPO_ERR_UNSUPPORTED;
     if ((reinterpret_cast<uintptr_t>(H) & 15u) || (reinterpret_cast<uintptr_t>(W) & 15u))
       return GRPO_ERR_INVALID_ARG;
   } else if (dtype == GRPO_F32) {

@@ -84,13 +84,13 @@ __device__ __forceinline__ Dims role_dims(const GemmArgs& a, int num_tiles) {
     d.num_m = num_tiles;
     d.num_n = (a.vc_len + BN - 1) / BN;
     d.num_kb = (ROLE == ROLE_DZ_KL ? 2 : 1) * (a.d / BK);
-  } else if (ROLE == ROLE_DH) {
+  } else if (ROLE == ROLE_DH) {   // d % 64 == 0: the last column tile may be partial
     d.num_m = num_tiles;
-    d.num_n = a.d / BN;
+    d.num_n = (a.d + BN - 1) / BN;
     d.num_kb = (a.vc_len + BK - 1) / BK;
   } else {
     d.num_m = (a.vc_len + BM - 1) / BM;
-    d.num_n = a.d / BN;
+    d.num_n = (a.d + BN - 1) / BN;
     d.num_kb = num_tiles * (BM / BK);
   }
   return d;
@@ -760,7 +760,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
         const int col = n * BN + c * 32;
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
-        if (!rv) continue;
+        if (!rv || col >= a.d) continue;   // columns past d (a partial last tile) hold zeros
         float* acc_row = a.dH_acc + (static_cast<size_t>(m_load) * BM + r) * a.d + col;
         if (a.dh_mode == 2 || a.dh_mode == 3) {
 #pragma unroll
@@ -807,7 +807,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
       for (int c = 0; c < BN / 32; ++c) {
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
-        if (!rv) continue;
+        if (!rv || n * BN + c * 32 >= a.d) continue;   // columns past d: a partial last tile
         if (empty_k) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) x[j] = 0.f;

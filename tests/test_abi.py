@@ -44,8 +44,8 @@ def test_host_validation_rejects_before_launch(lib):
                             1 << 20, nul)
     assert st == -1
     fake = ctypes.c_void_p(1 << 20)      # never dereferenced: validation fails first
-    # d not a multiple of 256 is unsupported on the bf16 tensor-core path
-    st = lib.grpo_score_fwd(fake, fake, 1, fake, fake, 4, 64, 320, 512, fake, fake, fake, fake,
+    # d not a multiple of 64 is unsupported on the bf16 tensor-core path
+    st = lib.grpo_score_fwd(fake, fake, 1, fake, fake, 4, 64, 288, 512, fake, fake, fake, fake,
                             fake, fake, 1 << 30, nul)
     assert st == -2
     # misaligned workspace

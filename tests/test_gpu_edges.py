@@ -1,6 +1,7 @@
 """Edge cases of the CUDA path against the oracle: a single token, V < 256 and V not a multiple
-of 32, T just past a tile boundary, the smallest bf16 hidden size, a completion with no scored
-token, an all-masked batch, groups of one, and a data-parallel normaliser override."""
+of 32, T just past a tile boundary, the smallest bf16 hidden size, hidden sizes that are not a
+multiple of 256, a completion with no scored token, an all-masked batch, groups of one, and a
+data-parallel normaliser override."""
 import numpy as np
 import pytest
 import torch
@@ -20,6 +21,10 @@ EDGES = {
     "v200_d256": W_("v200_d256", 1, (3,), 70, 1, 70, 256, 200),
     "v1000_t129": W_("v1000_t129", 2, (2,), 129, 100, 129, 512, 1000),
     "v257_t257_g1": W_("v257_t257_g1", 3, (1, 2), 257, 1, 257, 768, 257),
+    # hidden sizes that are multiples of 64 but not of 256: the last 256-column tile of dH and
+    # dW is partial (64 and 128 valid columns)
+    "d320_v1000": W_("d320_v1000", 2, (3,), 150, 20, 150, 320, 1000),
+    "d896_v3001": W_("d896_v3001", 1, (4,), 140, 40, 140, 896, 3001),
     "f32_v33": W_("f32_v33", 2, (2,), 9, 1, 9, 48, 33, dtype="f32"),
 }
 
@@ -63,3 +68,28 @@ def test_normaliser_override_for_data_parallel_shards(agg):
     g = run_gpu(b, old, ref, 0.2, 0.2, 0.04, agg=agg, norm=norm)
     o = run_oracle(b, old, ref, 0.2, 0.2, 0.04, agg=agg, norm=norm)
     print(compare(b, g, o))
+
+
+def test_partial_hidden_tile_chunked_backward_and_every_tile_mode():
+    """d = 576 = 2*256 + 64: three output column tiles of dH and dW, the last with 64 valid
+    columns, an odd count (so in tile mode 4 the second CTA of the last cluster has no column
+    tile of its own). A 3-chunk backward (V = 2600 in chunks of 1024) accumulates dH across
+    chunks through the partial tile. Every tile mode meets the parity bar; modes 2-4 are bitwise
+    equal to mode 0."""
+    from paper_2510_17158_gb300 import grpo as G
+    b = make_batch_numpy(W_("d576_v2600", 1, (4,), 160, 40, 160, 576, 2600))
+    old, ref = oracle_inputs(b)
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
+    print("chunked", compare(b, run_gpu(b, old, ref, 0.2, 0.2, 0.04, vocab_chunk=1024), o))
+    prev = G.grpo_get_tile_mode()
+    try:
+        outs = {}
+        for mode in (0, 1, 2, 3, 4):
+            G.grpo_set_tile_mode(mode)
+            outs[mode] = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+            print("mode", mode, compare(b, outs[mode], o))
+    finally:
+        G.grpo_set_tile_mode(prev)
+    for mode in (2, 3, 4):
+        for k in ("logp", "lse", "entropy", "argmax", "dH", "dW"):
+            assert torch.equal(outs[mode][k], outs[0][k]), (mode, k)

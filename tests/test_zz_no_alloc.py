@@ -30,8 +30,10 @@ def _inputs(seed, **over):
 
 def test_static_scratch_forward_matches_workspace_forward_twice():
     batches = [_inputs(11, prompts=1, T=260, len_lo=60, len_hi=260),
-               _inputs(12, prompts=1, group_sizes=(5,), T=140, len_lo=20, len_hi=140)]
-    for H, W, tok, mask in batches:                   # two calls in a row, different shapes
+               _inputs(12, prompts=1, group_sizes=(5,), T=140, len_lo=20, len_hi=140),
+               _inputs(13, prompts=1, group_sizes=(3,), T=100, len_lo=20, len_hi=100, d=320,
+                       V=1000)]                       # d a multiple of 64, not of 256
+    for H, W, tok, mask in batches:                   # calls in a row, different shapes
         S, T, d = H.shape
         ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
         ref = G.grpo_score_fwd(H, W, tok, mask, ws)
