@@ -69,3 +69,26 @@ def test_host_validation_rejects_before_launch(lib):
     assert st == -1
     st = lib.group_advantages(fake, fake, 2, 8, 0, 1e-4, fake, nul, 1024, nul)
     assert st == -4
+
+
+def test_process_wide_settings_validate_and_round_trip(lib):
+    """Host-only setters (no GPU work): tile mode 0-4 accepted and read back, others refused;
+    the progress window refuses negative values and a checkpoint with lag 0; the CTA-pair switch
+    maps to tile modes 1 / 0."""
+    prev = lib.grpo_get_tile_mode()
+    try:
+        for mode in (0, 1, 2, 3, 4):
+            assert lib.grpo_set_tile_mode(mode) == 0
+            assert lib.grpo_get_tile_mode() == mode
+        for bad in (-1, 5, 1 << 20):
+            assert lib.grpo_set_tile_mode(bad) == -1
+            assert lib.grpo_get_tile_mode() == 4          # unchanged by a refused call
+        assert lib.grpo_set_cta_pair(1) == 0 and lib.grpo_get_tile_mode() == 1
+        assert lib.grpo_set_cta_pair(0) == 0 and lib.grpo_get_tile_mode() == 0
+    finally:
+        lib.grpo_set_tile_mode(prev)
+    assert lib.grpo_set_gemm_window(-1, 2) == -1
+    assert lib.grpo_set_gemm_window(16, -1) == -1
+    assert lib.grpo_set_gemm_window(16, 0) == -1
+    assert lib.grpo_set_gemm_window(16, 4) == 0
+    assert lib.grpo_set_gemm_window(0, 0) == 0
