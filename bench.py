@@ -43,6 +43,13 @@ TILE_MODES = {0: "single CTA 128x256 (cta_group::1)",
               3: "4-CTA cluster, four 128x256 tiles sharing B by TMA multicast (cta_group::1)",
               4: "2-CTA cluster, two 128x256 tiles sharing A by TMA multicast (cta_group::1)"}
 
+def tiles_desc(G):
+    modes = [G.grpo_get_role_tile_mode(r) for r in range(4)]
+    if len(set(modes)) == 1:
+        return TILE_MODES[modes[0]]
+    return "; ".join(f"{role}: {TILE_MODES[m]}" for role, m in zip(("fwd", "dz", "dH", "dW"), modes))
+
+
 def peaks():
     try:
         p = json.load(open(PEAKS_PATH))
@@ -153,17 +160,21 @@ def kernel_source_sha() -> str:
     return hashlib.sha256(txt.encode()).hexdigest()[:16]
 
 
-def ncu_traffic(kernel: str, workload: str):
+def ncu_traffic(kernel: str, workload: str, tile_mode: int):
     """DRAM bytes per launch from a committed ncu summary of this kernel, if it was taken on the
-    current kernel source (profiles/<kernel>__<workload>.md with 'source_sha' and
-    'dram_bytes_per_launch_full' lines)."""
+    current kernel source in the tile mode the kernel runs in now (profiles/<kernel>__<workload>.md
+    with 'source_sha', 'tile_mode' and 'dram_bytes_per_launch_full' lines; a summary without a
+    'tile_mode' line was taken with single-CTA tiles)."""
     path = os.path.join(PROFILES, f"{kernel}__{workload}.md")
     if not os.path.exists(path):
         return None
     txt = open(path).read()
     sha = re.search(r"source_sha:\s*([0-9a-f]+)", txt)
     val = re.search(r"dram_bytes_per_launch_full:\s*([0-9.eE+]+)", txt)
+    mode = re.search(r"tile_mode:\s*(-?[0-9]+)", txt)
     if not sha or not val or sha.group(1) != kernel_source_sha():
+        return None
+    if (int(mode.group(1)) if mode else 0) != tile_mode:
         return None
     return float(val.group(1))
 
@@ -242,6 +253,12 @@ def run_gpu(args):
     from paper_2510_17158_gb300 import grpo as G
     from paper_2510_17158_gb300.synthetic import WORKLOADS, lm_head_flops, make_batch_torch
     G.grpo_set_tile_mode(args.tile_mode)
+    if args.role_tile_modes:
+        role_modes = [int(x) for x in args.role_tile_modes.split(",")]
+        if len(role_modes) != 4:
+            raise SystemExit("--role-tile-modes wants four comma-separated modes (fwd,dz,dH,dW)")
+        for role, m in enumerate(role_modes):
+            G.grpo_set_role_tile_mode(role, m)
     win = [int(x) for x in args.gemm_window.split(",")]
     G.grpo_set_gemm_window(win[0], win[1])
     w = apply_scale(WORKLOADS[args.config], args.scale)
@@ -399,7 +416,9 @@ def run_gpu(args):
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
                 "frac": round(achieved / pk["bf16_sustained"], 4),
                 "peak_source": f"{pk['source']} bf16 sustained (kernel timed inside a long step)",
-                "traffic": ncu_traffic(dom, w.name)}
+                # committed ncu summaries cover the GRPO path's own GEMMs
+                "traffic": (ncu_traffic(dom, w.name, G.grpo_get_role_tile_mode(GEMM_KERNELS.index(dom)))
+                            if args.path == "grpo" and not args.vocab_chunk else None)}
     else:
         roof = {"kernel": dom, "bound": "hbm", "achieved": None, "peak": pk["hbm_gbs"],
                 "unit": "GB/s", "frac": None, "traffic": None}
@@ -419,7 +438,7 @@ def run_gpu(args):
         "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
                    "d": d, "V": V, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
-                   "tiles": TILE_MODES[args.tile_mode],
+                   "tiles": tiles_desc(G),
                    "gemm_window": ("off" if win[0] == 0 else
                                    f"{win[0]} k-blocks, lag {win[1]} checkpoints"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
@@ -463,8 +482,13 @@ def main():
     ap.add_argument("--path", default="grpo", choices=["grpo", "sft", "grpo-exact-kl"],
                     help="grpo: the GRPO update (default); sft: the distillation loss step; "
                          "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
-    ap.add_argument("--tile-mode", type=int, default=0, choices=sorted(TILE_MODES),
-                    help="tensor-core tiles: " + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items()))
+    ap.add_argument("--tile-mode", type=int, default=-1, choices=[-1] + sorted(TILE_MODES),
+                    help="tensor-core tiles of every GEMM: -1 = the library's per-GEMM default "
+                         "(fwd 2, dz 0, dH 0, dW 4); "
+                         + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items()))
+    ap.add_argument("--role-tile-modes", default="",
+                    help="per-GEMM tile modes fwd,dz,dH,dW, applied after --tile-mode "
+                         "(-1 = that GEMM's default)")
     ap.add_argument("--gemm-window", default="0,0",
                     help="GEMM progress window CHECK,LAG: producers stay within LAG checkpoints of "
                          "CHECK k-blocks of the launch's average ('0,0' = off)")

@@ -252,11 +252,12 @@ int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms);
  * such a call are undefined. Process-wide; not for production use. */
 int grpo_debug_inject_stall(int32_t on);
 
-/* Tensor-core tile mode of the LM-head GEMMs, process-wide, for launches made afterwards (the
- * exact-KL GEMMs always use mode 0). Every mode computes the same 128-row output tiles with the
- * same summation order inside a tile; modes 0, 2, 3 and 4 issue identical MMAs and give bitwise
- * identical results, mode 1 (M = 256 MMAs) agrees within rounding.
- *   GRPO_TILE_SINGLE     (0, default): one CTA per 128 x 256 tile (tcgen05 cta_group::1).
+/* Tensor-core tile mode of the four LM-head GEMM roles, process-wide, for launches made
+ * afterwards (the exact-KL GEMMs always use single-CTA tiles). Every mode computes the same
+ * 128-row output tiles with the same summation order inside a tile; modes 0, 2, 3 and 4 issue
+ * identical MMAs and give bitwise identical results in any mix over the roles, and mode 1
+ * (M = 256 MMAs) agrees within rounding.
+ *   GRPO_TILE_SINGLE     (0): one CTA per 128 x 256 tile (tcgen05 cta_group::1).
  *   GRPO_TILE_CTA_PAIR   (1): clusters of two CTAs on one TPC compute 256 x 256 tiles with
  *                        cta_group::2, each CTA staging half of B.
  *   GRPO_TILE_MULTICAST  (2): clusters of two CTAs compute two 128 x 256 tiles that share a B
@@ -265,20 +266,34 @@ int grpo_debug_inject_stall(int32_t on);
  *   GRPO_TILE_MULTICAST_A (4): clusters of two CTAs compute the tiles of one row tile and two
  *                        adjacent column tiles, which share an A tile; each CTA loads half of
  *                        its rows and TMA multicast writes them to both.
- * Mode 0 is the default: on a power-capped GB300 it spends the least energy per flop of these
- * (the step's throughput is bounded by the power cap, so energy per flop sets it).
- * Returns GRPO_ERR_INVALID_ARG for any other mode. grpo_set_cta_pair(on) is mode 1 if on != 0,
- * else mode 0; grpo_get_tile_mode returns the current mode. */
+ *   GRPO_TILE_DEFAULT   (-1): the library's per-role choice, in force at load: the forward
+ *                        product in mode 2, the dz recompute and dH in mode 0, dW in mode 4 --
+ *                        the fastest mix measured on a power-capped GB300 (where the step's
+ *                        throughput is bounded by energy per flop, and operand re-reads from
+ *                        HBM cost energy).
+ * Roles: GRPO_ROLE_FWD (forward scoring product), GRPO_ROLE_DZ (its recompute into dz),
+ * GRPO_ROLE_DH, GRPO_ROLE_DW.
+ * grpo_set_tile_mode(m) puts every role in mode m (m = -1: each role's default);
+ * grpo_set_role_tile_mode(r, m) sets one role (m = -1: that role's default).
+ * grpo_get_tile_mode returns the mode all four roles share, or -1 when they differ (as they do
+ * by default); grpo_get_role_tile_mode returns the mode role r runs in.
+ * grpo_set_cta_pair(on) is grpo_set_tile_mode(on ? 1 : 0).
+ * Setters return GRPO_ERR_INVALID_ARG, changing nothing, for a mode outside -1..4 or a role
+ * outside 0..3; grpo_get_role_tile_mode returns GRPO_ERR_INVALID_ARG for such a role. */
 enum {
+  GRPO_TILE_DEFAULT = -1,
   GRPO_TILE_SINGLE = 0,
   GRPO_TILE_CTA_PAIR = 1,
   GRPO_TILE_MULTICAST = 2,
   GRPO_TILE_MULTICAST4 = 3,
   GRPO_TILE_MULTICAST_A = 4
 };
+enum { GRPO_ROLE_FWD = 0, GRPO_ROLE_DZ = 1, GRPO_ROLE_DH = 2, GRPO_ROLE_DW = 3 };
 int grpo_set_tile_mode(int32_t mode);
 int grpo_get_tile_mode(void);
 int grpo_set_cta_pair(int32_t on);
+int grpo_set_role_tile_mode(int32_t role, int32_t mode);
+int grpo_get_role_tile_mode(int32_t role);
 
 /* Progress window of the tensor-core GEMMs, process-wide, for launches made afterwards. Every
  * `check_kblocks` k-blocks of 64 the TMA producer of each CTA waits (at most 0.5 ms) until the

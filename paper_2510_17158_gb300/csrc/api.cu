@@ -31,7 +31,16 @@ struct EventPair {
 std::mutex g_mu;
 std::atomic<int> g_timing{0};
 std::atomic<int> g_inject_stall{0};
-std::atomic<int> g_tile_mode{GRPO_TILE_SINGLE};  // tensor-core tile mode (GRPO_TILE_*)
+// Tensor-core tile mode (GRPO_TILE_*) of each LM-head GEMM role, GRPO_ROLE_FWD .. GRPO_ROLE_DW.
+// Defaults, measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
+// V = 151936 (same box, back to back): the forward product shares its W tile between two
+// consecutive row tiles (B multicast, 323 -> 305 ms) and dW shares its dz^T tile between two
+// adjacent column tiles (A multicast, 344 -> 333 ms); the dz recompute and dH gain nothing from
+// either and keep single-CTA tiles.
+constexpr int kRoleDefault[4] = {GRPO_TILE_MULTICAST, GRPO_TILE_SINGLE, GRPO_TILE_SINGLE,
+                                 GRPO_TILE_MULTICAST_A};
+std::atomic<int> g_role_mode[4] = {{kRoleDefault[0]}, {kRoleDefault[1]}, {kRoleDefault[2]},
+                                   {kRoleDefault[3]}};
 std::atomic<int> g_win_check{0}, g_win_lag{0};  // GEMM progress window (k-blocks, checkpoints)
 std::atomic<long long> g_launches[GRPO_K_COUNT];
 std::vector<EventPair> g_pending[GRPO_K_COUNT];
@@ -739,18 +748,35 @@ int grpo_debug_inject_stall(int32_t on) {
   return GRPO_OK;
 }
 
-int grpo_set_cta_pair(int32_t on) {
-  g_tile_mode.store(on ? 1 : 0);
-  return GRPO_OK;
-}
-
 int grpo_set_tile_mode(int32_t mode) {
-  if (mode < GRPO_TILE_SINGLE || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
-  g_tile_mode.store(mode);
+  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
+  for (int r = GRPO_ROLE_FWD; r <= GRPO_ROLE_DW; ++r)
+    g_role_mode[r].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[r] : mode);
   return GRPO_OK;
 }
 
-int grpo_get_tile_mode(void) { return g_tile_mode.load(); }
+int grpo_set_cta_pair(int32_t on) {
+  return grpo_set_tile_mode(on ? GRPO_TILE_CTA_PAIR : GRPO_TILE_SINGLE);
+}
+
+int grpo_get_tile_mode(void) {
+  const int m = g_role_mode[GRPO_ROLE_FWD].load();
+  for (int r = GRPO_ROLE_DZ; r <= GRPO_ROLE_DW; ++r)
+    if (g_role_mode[r].load() != m) return GRPO_TILE_DEFAULT;   // roles differ
+  return m;
+}
+
+int grpo_set_role_tile_mode(int32_t role, int32_t mode) {
+  if (role < GRPO_ROLE_FWD || role > GRPO_ROLE_DW) return GRPO_ERR_INVALID_ARG;
+  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
+  g_role_mode[role].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[role] : mode);
+  return GRPO_OK;
+}
+
+int grpo_get_role_tile_mode(int32_t role) {
+  if (role < GRPO_ROLE_FWD || role > GRPO_ROLE_DW) return GRPO_ERR_INVALID_ARG;
+  return gemm_role_tile_mode(role);
+}
 
 int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag) {
   if (check_kblocks < 0 || lag < 0 || (check_kblocks > 0 && lag == 0)) return GRPO_ERR_INVALID_ARG;
@@ -768,8 +794,8 @@ void gemm_window_config(GemmArgs& a) {
 }
 
 int gemm_role_tile_mode(int role) {
-  (void)role;   // one process-wide mode for the four GEMM roles
-  return g_tile_mode.load();
+  // the exact-KL roles always run single-CTA tiles
+  return (role >= ROLE_FWD && role <= ROLE_DW) ? g_role_mode[role].load() : GRPO_TILE_SINGLE;
 }
 }  // namespace grpo
 

@@ -13,9 +13,10 @@
 // (bf16 in, f32 accumulate in tensor memory), warps 2-5 read the accumulator back with
 // tcgen05.ld (one TMEM lane = one output row per thread) and run the role's epilogue. Two
 // 256-column accumulators in TMEM let the epilogue of one tile overlap the MMAs of the next.
-// Tile modes (see Cfg): one CTA per 128 x 256 tile (cta_group::1, the default), a CTA pair per
-// 256 x 256 tile (cta_group::2), or 2- / 4-CTA clusters whose CTAs share one operand tile by
-// TMA multicast. Every wait is bounded (see mbar_wait_bounded).
+// Tile modes (see Cfg): one CTA per 128 x 256 tile (cta_group::1), a CTA pair per 256 x 256
+// tile (cta_group::2), or 2- / 4-CTA clusters whose CTAs share one operand tile by TMA
+// multicast; the host picks one per role (by default B multicast for FWD, A multicast for DW,
+// single CTA for DZ and DH). Every wait is bounded (see mbar_wait_bounded).
 #include <cfloat>
 
 #include "common.cuh"

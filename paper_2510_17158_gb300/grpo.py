@@ -63,6 +63,8 @@ def _declare(lib):
         "grpo_set_cta_pair": (ctypes.c_int, [_i32]),
         "grpo_set_tile_mode": (ctypes.c_int, [_i32]),
         "grpo_get_tile_mode": (ctypes.c_int, []),
+        "grpo_set_role_tile_mode": (ctypes.c_int, [_i32, _i32]),
+        "grpo_get_role_tile_mode": (ctypes.c_int, [_i32]),
         "grpo_set_gemm_window": (ctypes.c_int, [_i32, _i32]),
         "grpo_sft_loss_bwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p,
                                              _p, _p, _i32, _f64, _p, _p, _p, _p, _sz, _p]),
@@ -474,17 +476,34 @@ def grpo_set_cta_pair(on: bool):
     _check(_lib().grpo_set_cta_pair(1 if on else 0), "grpo_set_cta_pair")
 
 
+TILE_DEFAULT = -1
 TILE_SINGLE, TILE_CTA_PAIR, TILE_MULTICAST, TILE_MULTICAST4, TILE_MULTICAST_A = 0, 1, 2, 3, 4
+ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW = 0, 1, 2, 3
 
 
 def grpo_set_tile_mode(mode: int):
-    """0 single-CTA tiles (default), 1 CTA pairs (cta_group::2), 2 / 3 B tile shared by TMA
-    multicast in clusters of 2 / 4 CTAs, 4 A tile shared by TMA multicast in 2-CTA clusters."""
+    """Every GEMM role in one mode: 0 single-CTA tiles, 1 CTA pairs (cta_group::2), 2 / 3 B
+    tile shared by TMA multicast in clusters of 2 / 4 CTAs, 4 A tile shared by TMA multicast in
+    2-CTA clusters; -1 (TILE_DEFAULT) restores each role's default."""
     _check(_lib().grpo_set_tile_mode(int(mode)), "grpo_set_tile_mode")
 
 
 def grpo_get_tile_mode() -> int:
+    """The mode all four roles share, or -1 when they differ (as by default)."""
     return int(_lib().grpo_get_tile_mode())
+
+
+def grpo_set_role_tile_mode(role: int, mode: int):
+    """Tile mode of one GEMM role (ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW); -1 restores the
+    role's default."""
+    _check(_lib().grpo_set_role_tile_mode(int(role), int(mode)), "grpo_set_role_tile_mode")
+
+
+def grpo_get_role_tile_mode(role: int) -> int:
+    m = int(_lib().grpo_get_role_tile_mode(int(role)))
+    if m < 0:
+        raise ValueError(f"grpo_get_role_tile_mode: bad role {role}")
+    return m
 
 
 def grpo_set_gemm_window(check_kblocks: int, lag: int):

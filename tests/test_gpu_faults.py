@@ -20,26 +20,32 @@ def _small():
 
 
 def test_stalled_pipeline_times_out_and_context_survives():
+    """Single-CTA tiles (mode 0): CTA 0 leaves its first pipeline stage unfilled, its MMA wait
+    runs out, and the next call on the same context is bitwise correct."""
     b, (H, W, tok, mask) = _small()
     S, T, d = H.shape
     ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
-    good = G.grpo_score_fwd(H, W, tok, mask, ws)
-    torch.cuda.synchronize()
-    good = {k: v.clone() for k, v in good.items()}
-    assert G.grpo_last_device_error(ws)[0] == 0
-    G.grpo_debug_inject_stall(True)
+    G.grpo_set_tile_mode(G.TILE_SINGLE)
     try:
-        G.grpo_score_fwd(H, W, tok, mask, ws)
-        st, where = G.grpo_last_device_error(ws)       # synchronises; the kernel gave up
+        good = G.grpo_score_fwd(H, W, tok, mask, ws)
+        torch.cuda.synchronize()
+        good = {k: v.clone() for k, v in good.items()}
+        assert G.grpo_last_device_error(ws)[0] == 0
+        G.grpo_debug_inject_stall(True)
+        try:
+            G.grpo_score_fwd(H, W, tok, mask, ws)
+            st, where = G.grpo_last_device_error(ws)       # synchronises; the kernel gave up
+        finally:
+            G.grpo_debug_inject_stall(False)
+        assert st == TIMEOUT, (st, where)
+        assert where // 16 == 3                              # recorded by a GEMM wait
+        again = G.grpo_score_fwd(H, W, tok, mask, ws)
+        torch.cuda.synchronize()
+        assert G.grpo_last_device_error(ws)[0] == 0
+        for k in ("logp", "lse", "entropy", "argmax", "valid_count"):
+            assert torch.equal(again[k], good[k]), k
     finally:
-        G.grpo_debug_inject_stall(False)
-    assert st == TIMEOUT, (st, where)
-    assert where // 16 == 3                              # recorded by a GEMM wait
-    again = G.grpo_score_fwd(H, W, tok, mask, ws)
-    torch.cuda.synchronize()
-    assert G.grpo_last_device_error(ws)[0] == 0
-    for k in ("logp", "lse", "entropy", "argmax", "valid_count"):
-        assert torch.equal(again[k], good[k]), k
+        G.grpo_set_tile_mode(G.TILE_DEFAULT)
 
 
 def test_token_out_of_range_sets_status():

@@ -126,8 +126,9 @@ def test_tile_modes_match_oracle_and_single_cta_tiles(name):
     b = _batch(name)
     old, ref = oracle_inputs(b)
     o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
-    prev = G.grpo_get_tile_mode()
-    assert prev == G.TILE_SINGLE                     # the library's default
+    # the library's per-role defaults: forward B-multicast, dz and dH single CTA, dW A-multicast
+    assert [G.grpo_get_role_tile_mode(r) for r in range(4)] == [2, 0, 0, 4]
+    assert G.grpo_get_tile_mode() == G.TILE_DEFAULT
     try:
         G.grpo_set_tile_mode(G.TILE_SINGLE)
         g0 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
@@ -145,13 +146,49 @@ def test_tile_modes_match_oracle_and_single_cta_tiles(name):
                     assert torch.equal(g[k], g0[k]), (mode, k)
                 assert g["loss"] == g0["loss"]
     finally:
-        G.grpo_set_tile_mode(prev)
+        G.grpo_set_tile_mode(G.TILE_DEFAULT)
+
+
+@pytest.mark.parametrize("name", ["d2048_v32k"])
+def test_mixed_role_tile_modes_bitwise_equal_single_cta(name):
+    """Each GEMM role may run in its own tile mode (grpo_set_role_tile_mode). Mixes of modes 0,
+    2, 3 and 4 issue the same MMAs per tile as mode 0 everywhere, so the forward statistics, the
+    recomputed dz and both gradients are bitwise equal to all-mode-0 outputs; a mix with the CTA
+    pair for the recompute only (lse from single-CTA tiles, z recomputed by M = 256 MMAs) agrees
+    with the oracle within the parity bar."""
+    from paper_2510_17158_gb300 import grpo as G
+    b = _batch(name)
+    old, ref = oracle_inputs(b)
+    o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
+    try:
+        G.grpo_set_tile_mode(G.TILE_SINGLE)
+        g0 = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+        G.grpo_set_tile_mode(G.TILE_DEFAULT)
+        g = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+        print("default roles", compare(b, g, o))
+        for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
+            assert torch.equal(g[k], g0[k]), ("default", k)
+        for mix in ((2, 2, 0, 0), (2, 3, 4, 0), (4, 0, 2, 3)):
+            for role, m in enumerate(mix):
+                G.grpo_set_role_tile_mode(role, m)
+            assert [G.grpo_get_role_tile_mode(r) for r in range(4)] == list(mix)
+            g = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+            print("roles", mix, compare(b, g, o))
+            for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
+                assert torch.equal(g[k], g0[k]), (mix, k)
+            assert g["loss"] == g0["loss"]
+        for role, m in enumerate((0, 1, 0, 0)):
+            G.grpo_set_role_tile_mode(role, m)
+        g = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
+        print("roles (0, 1, 0, 0)", compare(b, g, o))      # compare() asserts the parity bar
+    finally:
+        G.grpo_set_tile_mode(G.TILE_DEFAULT)
 
 
 def test_tile_mode_rejects_unknown_modes():
     from paper_2510_17158_gb300 import grpo as G
     prev = G.grpo_get_tile_mode()
-    for bad in (-1, 5):
+    for bad in (-2, 5):
         with pytest.raises(G.GrpoError):
             G.grpo_set_tile_mode(bad)
     assert G.grpo_get_tile_mode() == prev
