@@ -798,7 +798,3 @@ int gemm_role_tile_mode(int role) {
   return (role >= ROLE_FWD && role <= ROLE_DW) ? g_role_mode[role].load() : GRPO_TILE_SINGLE;
 }
 }  // namespace grpo
-
-extern "C" {
-
-}  // extern "C"
