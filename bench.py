@@ -39,9 +39,7 @@ GEMM_KERNELS = ("fwd_gemm_tc", "bwd_dz_gemm_tc", "bwd_dh_gemm_tc", "bwd_dw_gemm_
 
 TILE_MODES = {0: "single CTA 128x256 (cta_group::1)",
               1: "CTA pair 256x256 (cta_group::2)",
-              2: "2-CTA cluster, two 128x256 tiles sharing B by TMA multicast (cta_group::1)",
-              3: "4-CTA cluster, four 128x256 tiles sharing B by TMA multicast (cta_group::1)",
-              4: "2-CTA cluster, two 128x256 tiles sharing A by TMA multicast (cta_group::1)"}
+              2: "CTA pair 256x512 (cta_group::2, two N=256 MMAs per k-step)"}
 
 def tiles_desc(G):
     modes = [G.grpo_get_role_tile_mode(r) for r in range(4)]
@@ -200,7 +198,7 @@ def run_reference(args, ws_size, rank):
     line = cpu_baseline(w, args.ref_tokens, steps=args.steps, warmup=args.warmup)
     value = line["value"]
     out = {"metric": "scored tokens/sec (fwd+bwd)", "value": value, "unit": "tokens/s",
-           "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+           "n_gpus": ws_size, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": line["ms_per_step"], "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
            "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": w.T,
@@ -210,6 +208,22 @@ def run_reference(args, ws_size, rank):
            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
+
+
+def blas_threads() -> int:
+    """Threads the oracle's numpy BLAS runs with (torch.distributed.run sets OMP_NUM_THREADS=1
+    in every rank unless the caller set it)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [p["num_threads"] for p in threadpool_info() if p.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return os.cpu_count()
 
 
 def cpu_baseline(w, n_tokens, steps=1, warmup=0):
@@ -238,9 +252,10 @@ def cpu_baseline(w, n_tokens, steps=1, warmup=0):
         if it >= warmup:
             times.append(time.perf_counter() - t0)
     per = sum(times) / len(times)
-    return {"value": n_tokens / per, "ms_per_step": per * 1e3, "cores": os.cpu_count(),
+    nthr = blas_threads()
+    return {"value": n_tokens / per, "ms_per_step": per * 1e3, "cores": nthr,
             "sample": f"{n_tokens} scored tokens of one completion, full d={d}, V={V} "
-                      f"(fwd + loss + dH + full dW), float64 numpy on {os.cpu_count()} host "
+                      f"(fwd + loss + dH + full dW), float64 numpy on {nthr} host "
                       f"threads; mean of {len(times)} run(s)"}
 
 
@@ -469,26 +484,29 @@ def run_gpu(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--gpus", type=int, default=1,
+                    help="GPUs (one process each); without WORLD_SIZE in the environment, N > 1 "
+                         "re-launches this command under torch.distributed.run")
+    ap.add_argument("--master-port", type=int, default=29533)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--vocab-chunk", type=int, default=0)
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-tokens", type=int, default=32)
     ap.add_argument("--ref-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--path", default="grpo", choices=["grpo", "sft", "grpo-exact-kl"],
                     help="grpo: the GRPO update (default); sft: the distillation loss step; "
                          "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
-    ap.add_argument("--tile-mode", type=int, default=-1, choices=[-1] + sorted(TILE_MODES),
+    ap.add_argument("--tile-mode", type=int, default=-1, choices=[-1, 0, 1],
                     help="tensor-core tiles of every GEMM: -1 = the library's per-GEMM default "
-                         "(fwd 2, dz 0, dH 0, dW 4); "
-                         + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items()))
+                         "(fwd 0, dz 0, dH 2, dW 2); "
+                         + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items() if k < 2))
     ap.add_argument("--role-tile-modes", default="",
                     help="per-GEMM tile modes fwd,dz,dH,dW, applied after --tile-mode "
-                         "(-1 = that GEMM's default)")
+                         "(-1 = that GEMM's default; 2 = " + TILE_MODES[2] + ", dH and dW only)")
     ap.add_argument("--gemm-window", default="0,0",
                     help="GEMM progress window CHECK,LAG: producers stay within LAG checkpoints of "
                          "CHECK k-blocks of the launch's average ('0,0' = off)")
@@ -501,7 +519,15 @@ def main():
     args = ap.parse_args()
     if args.impl == "ours":
         args.warmup = max(3, args.warmup)      # timing rule: at least 3 warm-up steps
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # one process per GPU: re-launch this command under torch.distributed.run
+        cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+               f"--nproc-per-node={args.gpus}", "--master-addr=127.0.0.1",
+               f"--master-port={args.master_port}", os.path.abspath(__file__)] + sys.argv[1:]
+        raise SystemExit(subprocess.call(cmd))
     ws_n, rank, _ = dist_env()
+    if ws_n != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={ws_n}")
     if args.impl == "reference":
         run_reference(args, ws_n, rank)
         return

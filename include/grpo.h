@@ -105,7 +105,12 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
  *    a multiple of 128) does not fit returns GRPO_ERR_WORKSPACE before anything is enqueued;
  *  - it allocates nothing and calls no allocating routine;
  *  - the first call made with a given device current looks up the array's device address
- *    (cudaGetSymbolAddress) and caches it: make that first call before any stream capture;
+ *    (cudaGetSymbolAddress) and caches it: make that first call before any stream capture (a
+ *    first call inside a capture returns GRPO_ERR_CUDA). Later calls whose stream is not being
+ *    captured look the address up again, so a context re-created by cudaDeviceReset is handled;
+ *    calls inside a capture use the cached address;
+ *  - its launches are counted by the kernel accounting below like those of grpo_score_fwd, and
+ *    grpo_debug_inject_stall applies to its tensor-core GEMM;
  *  - all calls share the one array and each overwrites it: calls that overlap on the GPU
  *    (different streams, or different host threads on one device) race and corrupt each
  *    other's results;
@@ -253,40 +258,35 @@ int grpo_timing_read(int32_t kernel_id, int64_t* launches, double* total_ms);
 int grpo_debug_inject_stall(int32_t on);
 
 /* Tensor-core tile mode of the four LM-head GEMM roles, process-wide, for launches made
- * afterwards (the exact-KL GEMMs always use single-CTA tiles). Every mode computes the same
- * 128-row output tiles with the same summation order inside a tile; modes 0, 2, 3 and 4 issue
- * identical MMAs and give bitwise identical results in any mix over the roles, and mode 1
- * (M = 256 MMAs) agrees within rounding.
- *   GRPO_TILE_SINGLE     (0): one CTA per 128 x 256 tile (tcgen05 cta_group::1).
- *   GRPO_TILE_CTA_PAIR   (1): clusters of two CTAs on one TPC compute 256 x 256 tiles with
- *                        cta_group::2, each CTA staging half of B.
- *   GRPO_TILE_MULTICAST  (2): clusters of two CTAs compute two 128 x 256 tiles that share a B
- *                        tile; each CTA loads half of it and TMA multicast writes it to both.
- *   GRPO_TILE_MULTICAST4 (3): the same with clusters of four CTAs, each loading a quarter of B.
- *   GRPO_TILE_MULTICAST_A (4): clusters of two CTAs compute the tiles of one row tile and two
- *                        adjacent column tiles, which share an A tile; each CTA loads half of
- *                        its rows and TMA multicast writes them to both.
- *   GRPO_TILE_DEFAULT   (-1): the library's per-role choice, in force at load: the forward
- *                        product in mode 2, the dz recompute and dH in mode 0, dW in mode 4 --
- *                        the fastest mix measured on a power-capped GB300 (where the step's
- *                        throughput is bounded by energy per flop, and operand re-reads from
- *                        HBM cost energy).
+ * afterwards (the exact-KL GEMMs always use single-CTA tiles). Every mode sums each output
+ * element over K in the same k-block order; modes 1 and 2 issue the same M = 256 MMAs and give
+ * bitwise identical dH and dW, and agree with mode 0 (M = 128 MMAs) within rounding. Every TMA
+ * copy lands in the issuing CTA's own shared memory (no multicast).
+ *   GRPO_TILE_SINGLE        (0): one CTA per 128 x 256 tile (tcgen05 cta_group::1), two TMEM
+ *                           accumulators (a tile's epilogue overlaps the next tile's MMAs).
+ *   GRPO_TILE_CTA_PAIR      (1): clusters of two CTAs on one TPC compute 256 x 256 tiles with
+ *                           cta_group::2, each CTA staging its 128 rows of A and half of B.
+ *   GRPO_TILE_CTA_PAIR_WIDE (2): dH and dW only. The CTA pair computes 256 x 512 tiles: two
+ *                           N = 256 MMAs per k-step into one 512-column accumulator, each CTA
+ *                           staging 128 rows of A and 256 rows of B per k-block, i.e. half of
+ *                           mode 0's operand bytes per flop.
+ *   GRPO_TILE_DEFAULT      (-1): the library's per-role choice, in force at load: the forward
+ *                           product and the dz recompute in mode 0, dH and dW in mode 2.
  * Roles: GRPO_ROLE_FWD (forward scoring product), GRPO_ROLE_DZ (its recompute into dz),
  * GRPO_ROLE_DH, GRPO_ROLE_DW.
- * grpo_set_tile_mode(m) puts every role in mode m (m = -1: each role's default);
- * grpo_set_role_tile_mode(r, m) sets one role (m = -1: that role's default).
+ * grpo_set_tile_mode(m) puts every role in mode m (m = -1: each role's default; m = 0 or 1);
+ * grpo_set_role_tile_mode(r, m) sets one role (m = -1: that role's default; m = 2 for GRPO_ROLE_DH
+ * and GRPO_ROLE_DW only).
  * grpo_get_tile_mode returns the mode all four roles share, or -1 when they differ (as they do
  * by default); grpo_get_role_tile_mode returns the mode role r runs in.
  * grpo_set_cta_pair(on) is grpo_set_tile_mode(on ? 1 : 0).
- * Setters return GRPO_ERR_INVALID_ARG, changing nothing, for a mode outside -1..4 or a role
- * outside 0..3; grpo_get_role_tile_mode returns GRPO_ERR_INVALID_ARG for such a role. */
+ * Setters return GRPO_ERR_INVALID_ARG, changing nothing, for a mode or role outside these
+ * ranges; grpo_get_role_tile_mode returns GRPO_ERR_INVALID_ARG for a role outside 0..3. */
 enum {
   GRPO_TILE_DEFAULT = -1,
   GRPO_TILE_SINGLE = 0,
   GRPO_TILE_CTA_PAIR = 1,
-  GRPO_TILE_MULTICAST = 2,
-  GRPO_TILE_MULTICAST4 = 3,
-  GRPO_TILE_MULTICAST_A = 4
+  GRPO_TILE_CTA_PAIR_WIDE = 2
 };
 enum { GRPO_ROLE_FWD = 0, GRPO_ROLE_DZ = 1, GRPO_ROLE_DH = 2, GRPO_ROLE_DW = 3 };
 int grpo_set_tile_mode(int32_t mode);

@@ -32,13 +32,12 @@ std::mutex g_mu;
 std::atomic<int> g_timing{0};
 std::atomic<int> g_inject_stall{0};
 // Tensor-core tile mode (GRPO_TILE_*) of each LM-head GEMM role, GRPO_ROLE_FWD .. GRPO_ROLE_DW.
-// Defaults, measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
-// V = 151936 (same box, back to back): the forward product shares its W tile between two
-// consecutive row tiles (B multicast, 323 -> 305 ms) and dW shares its dz^T tile between two
-// adjacent column tiles (A multicast, 344 -> 333 ms); the dz recompute and dH gain nothing from
-// either and keep single-CTA tiles.
-constexpr int kRoleDefault[4] = {GRPO_TILE_MULTICAST, GRPO_TILE_SINGLE, GRPO_TILE_SINGLE,
-                                 GRPO_TILE_MULTICAST_A};
+// The forward product and the dz recompute (K = d, a short reduction per tile) keep single-CTA
+// tiles, whose two accumulators overlap each tile's epilogue with the next tile's MMAs. dH and
+// dW (K = vocabulary / tokens: thousands of k-blocks per tile) take the 256 x 512 CTA-pair
+// tiles, which stage half of a single-CTA tile's operand bytes per flop.
+constexpr int kRoleDefault[4] = {GRPO_TILE_SINGLE, GRPO_TILE_SINGLE, GRPO_TILE_CTA_PAIR_WIDE,
+                                 GRPO_TILE_CTA_PAIR_WIDE};
 std::atomic<int> g_role_mode[4] = {{kRoleDefault[0]}, {kRoleDefault[1]}, {kRoleDefault[2]},
                                    {kRoleDefault[3]}};
 std::atomic<int> g_win_check{0}, g_win_lag{0};  // GEMM progress window (k-blocks, checkpoints)
@@ -78,6 +77,19 @@ int counted(int kid, cudaStream_t st, F&& launch) {
   g_launches[kid].fetch_add(1);
   return e == cudaSuccess ? GRPO_OK : GRPO_ERR_CUDA;
 }
+
+}  // namespace
+
+namespace grpo {
+int counted_launch(int kernel_id, cudaStream_t st, const std::function<cudaError_t()>& launch) {
+  if (kernel_id < 0 || kernel_id >= GRPO_K_COUNT) return GRPO_ERR_INVALID_ARG;
+  return counted(kernel_id, st, launch);
+}
+
+int debug_inject_stall() { return g_inject_stall.load(); }
+}  // namespace grpo
+
+namespace {
 
 #define GRPO_TRY(x)             \
   do {                          \
@@ -352,7 +364,7 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
   GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, valid_count, st));
   const int tm = gemm_role_tile_mode(ROLE_FWD);
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapW, W, d, V, d, gemm_b_box_rows(tm)))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
@@ -476,9 +488,9 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   if (mode == 2 && (!make_map(&mapHrk, v.hrp, d, L.rows_cap, d, kTileRows) ||
                     !make_map(&mapWrk, W_ref, d, V, d, kTileN)))
     return GRPO_ERR_CUDA;
-  if (!make_map(&mapHk, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+  if (!make_map(&mapHk, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapWk, W, d, V, d, gemm_b_box_rows(tm)) ||
-      !make_map(&mapDzK, dz, vc, L.rows_cap, vc, gemm_a_box_rows(tm_dh)) ||
+      !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
       !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
       !make_map(&mapHmn, v.hp, d, L.rows_cap, d, 64))
     return GRPO_ERR_CUDA;
@@ -624,7 +636,7 @@ int grpo_score_fwd_shard(const void* H, const void* W_shard, int32_t dtype,
   GRPO_TRY(pack_tokens(mask, S, T, d, H, L, v, v.counts, st));
   const int tm = gemm_role_tile_mode(ROLE_FWD);
   CUtensorMap mapH, mapW;
-  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, gemm_a_box_rows(tm)) ||
+  if (!make_map(&mapH, v.hp, d, L.rows_cap, d, kTileRows) ||
       !make_map(&mapW, W_shard, d, V_shard, d, gemm_b_box_rows(tm)))
     return GRPO_ERR_CUDA;
   GemmArgs a = base_args(L, v, S, T, d, V_shard, tokens, mask);
@@ -749,7 +761,8 @@ int grpo_debug_inject_stall(int32_t on) {
 }
 
 int grpo_set_tile_mode(int32_t mode) {
-  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
+  if (mode != GRPO_TILE_DEFAULT && mode != GRPO_TILE_SINGLE && mode != GRPO_TILE_CTA_PAIR)
+    return GRPO_ERR_INVALID_ARG;
   for (int r = GRPO_ROLE_FWD; r <= GRPO_ROLE_DW; ++r)
     g_role_mode[r].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[r] : mode);
   return GRPO_OK;
@@ -768,7 +781,10 @@ int grpo_get_tile_mode(void) {
 
 int grpo_set_role_tile_mode(int32_t role, int32_t mode) {
   if (role < GRPO_ROLE_FWD || role > GRPO_ROLE_DW) return GRPO_ERR_INVALID_ARG;
-  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_MULTICAST_A) return GRPO_ERR_INVALID_ARG;
+  const bool long_k = role == GRPO_ROLE_DH || role == GRPO_ROLE_DW;
+  if (mode != GRPO_TILE_DEFAULT && mode != GRPO_TILE_SINGLE && mode != GRPO_TILE_CTA_PAIR &&
+      !(long_k && mode == GRPO_TILE_CTA_PAIR_WIDE))
+    return GRPO_ERR_INVALID_ARG;
   g_role_mode[role].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[role] : mode);
   return GRPO_OK;
 }

@@ -7,8 +7,12 @@
 //
 // The scratch is one file-scope __device__ array of kStaticScratchBytes (64 MiB). Every GPU on
 // which this library is loaded keeps that array until the process exits. In host code the
-// array's name is only a host-side stand-in, so the device address is looked up once per device
-// with cudaGetSymbolAddress (on the first call made with that device current) and cached.
+// array's name is only a host-side stand-in, so its device address is looked up with
+// cudaGetSymbolAddress, with the device current, on the first call made on that device, and
+// cached. A call made while its stream is not being captured looks the address up again (cheap,
+// allocates nothing), so a context torn down and re-created (cudaDeviceReset) never leaves a
+// stale address behind; a call made during stream capture uses the cached address, which is why
+// the first call on a device must come before any capture.
 #include <cudaTypedefs.h>
 
 #include <cstring>
@@ -31,12 +35,15 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void* g_dev_ptr[kMaxDevices];  // device address of g_fwd_scratch, per device
 
-int scratch_address(void** out) {
+int scratch_address(cudaStream_t st, void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return GRPO_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return GRPO_ERR_UNSUPPORTED;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) return GRPO_ERR_CUDA;
   std::lock_guard<std::mutex> lk(g_mu);
-  if (g_dev_ptr[dev] == nullptr) {
+  if (g_dev_ptr[dev] == nullptr || cap == cudaStreamCaptureStatusNone) {
+    if (cap != cudaStreamCaptureStatusNone) return GRPO_ERR_CUDA;   // first call inside a capture
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_fwd_scratch) != cudaSuccess || p == nullptr)
       return GRPO_ERR_CUDA;
@@ -127,8 +134,9 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
   const StaticLayout L = static_layout(S, T, d, V, dtype);
   if (L.end > kStaticScratchBytes) return GRPO_ERR_WORKSPACE;  // batch too large for the array
 
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   void* base = nullptr;
-  const int st_addr = scratch_address(&base);
+  const int st_addr = scratch_address(st, &base);
   if (st_addr != GRPO_OK) return st_addr;
   char* b = static_cast<char*>(base);
   WsHeader* hdr = reinterpret_cast<WsHeader*>(b);
@@ -138,26 +146,32 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
   float* zy = reinterpret_cast<float*>(b + L.zy);
   float4* partials = reinterpret_cast<float4*>(b + L.partials);
   void* hp = b + L.hp;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
 
   // The array keeps the previous call's contents: the status word must start at zero. Every
   // other region used below is fully written before it is read within this call.
   int rc = ok_or_cuda(cudaMemsetAsync(hdr, 0, sizeof(WsHeader), st));
   if (rc != GRPO_OK) return rc;
-  rc = ok_or_cuda(launch_mask_scan(mask, S, T, valid_count, st));
+  rc = counted_launch(GRPO_K_MASK_SCAN, st,
+                      [&] { return launch_mask_scan(mask, S, T, valid_count, st); });
   if (rc != GRPO_OK) return rc;
   if (dtype == GRPO_F32) {
-    rc = ok_or_cuda(launch_f32_fwd(static_cast<const float*>(H), static_cast<const float*>(W),
-                                   tokens, mask, S, T, d, V, logp, lse, entropy, argmax, hdr, st));
+    rc = counted_launch(GRPO_K_F32_FWD, st, [&] {
+      return launch_f32_fwd(static_cast<const float*>(H), static_cast<const float*>(W), tokens,
+                            mask, S, T, d, V, logp, lse, entropy, argmax, hdr, st);
+    });
   } else {
-    rc = ok_or_cuda(launch_pack(mask, valid_count, S, T, L.rows_cap, seq_base, row_pos, pos_row,
-                                hdr, st));
+    rc = counted_launch(GRPO_K_PACK, st, [&] {
+      return launch_pack(mask, valid_count, S, T, L.rows_cap, seq_base, row_pos, pos_row, hdr,
+                         st);
+    });
     if (rc != GRPO_OK) return rc;
-    rc = ok_or_cuda(launch_gather_rows(H, d, row_pos, hdr, L.rows_cap, hp, st));
+    rc = counted_launch(GRPO_K_GATHER, st, [&] {
+      return launch_gather_rows(H, d, row_pos, hdr, L.rows_cap, hp, st);
+    });
     if (rc != GRPO_OK) return rc;
     const int tm = gemm_role_tile_mode(ROLE_FWD);
     CUtensorMap mapH, mapW;
-    if (!bf16_map(&mapH, hp, d, static_cast<uint64_t>(L.rows_cap), gemm_a_box_rows(tm)) ||
+    if (!bf16_map(&mapH, hp, d, static_cast<uint64_t>(L.rows_cap), kTileRows) ||
         !bf16_map(&mapW, W, d, V, gemm_b_box_rows(tm)))
       return GRPO_ERR_CUDA;
     GemmArgs a;
@@ -174,12 +188,16 @@ extern "C" int grpo_score_fwd_static(const void* H, const void* W, int32_t dtype
     a.num_strips = L.num_strips;
     a.partials = partials;
     a.zy = zy;
+    a.inject_stall = debug_inject_stall();
     gemm_window_config(a);
     const int grid = gemm_grid(L.max_tiles, L.num_strips, tm);
-    rc = ok_or_cuda(launch_gemm(ROLE_FWD, mapH, mapW, a, grid, tm, st));
+    rc = counted_launch(GRPO_K_FWD_GEMM, st,
+                        [&] { return launch_gemm(ROLE_FWD, mapH, mapW, a, grid, tm, st); });
     if (rc != GRPO_OK) return rc;
-    rc = ok_or_cuda(launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, pos_row,
-                                     tokens, mask, S, T, V, logp, lse, entropy, argmax, hdr, st));
+    rc = counted_launch(GRPO_K_FWD_MERGE, st, [&] {
+      return launch_fwd_merge(partials, L.rows_cap, L.num_strips, zy, pos_row, tokens, mask, S,
+                              T, V, logp, lse, entropy, argmax, hdr, st);
+    });
   }
   if (rc != GRPO_OK) return rc;
   if (status_out)

@@ -11,12 +11,13 @@
 //
 // Block = 6 warps: warp 0 issues TMA loads into a shared-memory ring, warp 1 issues tcgen05.mma
 // (bf16 in, f32 accumulate in tensor memory), warps 2-5 read the accumulator back with
-// tcgen05.ld (one TMEM lane = one output row per thread) and run the role's epilogue. Two
-// 256-column accumulators in TMEM let the epilogue of one tile overlap the MMAs of the next.
-// Tile modes (see Cfg): one CTA per 128 x 256 tile (cta_group::1), a CTA pair per 256 x 256
-// tile (cta_group::2), or 2- / 4-CTA clusters whose CTAs share one operand tile by TMA
-// multicast; the host picks one per role (by default B multicast for FWD, A multicast for DW,
-// single CTA for DZ and DH). Every wait is bounded (see mbar_wait_bounded).
+// tcgen05.ld (one TMEM lane = one output row per thread) and run the role's epilogue.
+// Tile modes (see Cfg): one CTA per 128 x 256 tile (cta_group::1) with two TMEM accumulators so
+// that the epilogue of one tile overlaps the MMAs of the next; a CTA pair per 256 x 256 tile
+// (cta_group::2, two accumulators); or, for the long-K roles DH and DW, a CTA pair per 256 x 512
+// tile (cta_group::2, two N = 256 MMAs per k-step into one 512-column accumulator). Every TMA
+// load lands in the issuing CTA's own shared memory (the pair modes count both CTAs' bytes on
+// the leader's barrier). Every wait is bounded (see mbar_wait_bounded).
 #include <cfloat>
 
 #include "common.cuh"
@@ -39,36 +40,36 @@ constexpr int NUM_THREADS = 192;
 constexpr int GROUP_M = GRPO_GROUP_M;      // raster: row units sharing each column sweep
 
 // Tile modes (MODE template parameter):
-//   0 single CTA : one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128).
+//   0 single CTA : one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128); two
+//                  256-column accumulators in TMEM.
 //   1 CTA pair   : a cluster of 2 CTAs on one TPC computes a 256 x 256 tile with cta_group::2
-//                  (M = 256): each CTA stages its 128 rows of A and half (128 rows) of B, so the
-//                  per-SM operand traffic for B halves and the ring can be 6 deep.
-//   2, 3 B multicast: a cluster of CL = 2 (mode 2) or 4 (mode 3) CTAs computes CL 128 x 256
-//                  tiles of consecutive row tiles that share their B tile, with cta_group::1
-//                  MMAs; each CTA loads 1/CL of B and TMA multicast delivers it to all of them,
-//                  so per-CTA L2 -> SM traffic drops from 48 KB to 16 + 32/CL KB per k-block and
-//                  the CTAs of a cluster read B in lockstep.
-//   4 A multicast: a cluster of 2 CTAs computes the 128 x 256 tiles of one row tile and two
-//                  adjacent column tiles, which share their A tile; each CTA loads half of A's
-//                  rows and TMA multicast delivers them to both, so one read of an A tile from
-//                  HBM or L2 serves two column tiles.
+//                  (M = 256): each CTA stages its 128 rows of A and half (128 rows) of B, and the
+//                  pair's tensor cores read both halves of B, so per-SM operand traffic per flop
+//                  is 2/3 of mode 0's and the ring can be 6 deep. Two accumulators.
+//   2 wide pair  : the CTA pair computes a 256 x 512 tile: per k-step two N = 256 MMAs write the
+//                  two 256-column halves of one 512-column accumulator. Each CTA stages 128 rows
+//                  of A and 2 x 128 rows of B per k-block (48 KB), i.e. half of mode 0's operand
+//                  bytes per flop. The epilogue does not overlap the next tile's MMAs, which is
+//                  negligible for the long-K roles DH and DW (the only roles this mode serves:
+//                  thousands of k-blocks per tile against one epilogue).
 template <int MODE>
 struct Cfg {
-  static constexpr int CL = MODE == 0 ? 1 : (MODE == 3 ? 4 : 2);      // CTAs per cluster
-  static constexpr bool MC_A = MODE == 4;                               // A shared by multicast
-  static constexpr bool MC_B = MODE == 2 || MODE == 3;                  // B shared by multicast
-  static constexpr uint16_t MASK = static_cast<uint16_t>((1u << CL) - 1u);
+  static constexpr bool PAIR = MODE != 0;                   // cta_group::2 on a 2-CTA cluster
+  static constexpr int CL = PAIR ? 2 : 1;                   // CTAs per cluster
+  static constexpr int NT = MODE == 2 ? 2 : 1;              // 256-column MMAs per k-step
+  static constexpr int ACC_BUFS = MODE == 2 ? 1 : 2;        // accumulators in TMEM
   static constexpr int STAGES = MODE == 1 ? 6 : 4;
-  static constexpr uint32_t A_STAGE = BM * BK * 2;                      // 16 KB
-  static constexpr uint32_t A_LOAD_ROWS = MC_A ? BM / CL : BM;          // A rows this CTA loads
-  static constexpr uint32_t B_ROWS = MODE == 1 ? BN / 2 : BN;           // B rows staged here
-  static constexpr uint32_t B_LOAD_ROWS =                               // B rows this CTA loads
-      MODE == 1 ? BN / 2 : (MC_B ? BN / CL : BN);
-  static constexpr uint32_t B_STAGE = B_ROWS * BK * 2;                  // 16 or 32 KB
-  static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;               // bytes landing per CTA
+  static constexpr uint32_t A_STAGE = BM * BK * 2;          // 16 KB
+  static constexpr uint32_t B_HALF_ROWS = PAIR ? BN / 2 : BN;   // B rows per MMA staged here
+  static constexpr uint32_t B_ROWS = NT * B_HALF_ROWS;      // B rows staged here per k-block
+  static constexpr uint32_t B_HALF_STAGE = B_HALF_ROWS * BK * 2;
+  static constexpr uint32_t B_STAGE = B_ROWS * BK * 2;      // 32, 16 or 32 KB
+  static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;   // bytes landing per CTA
   static constexpr size_t SMEM = size_t(STAGES) * STAGE_TX + 1024 + 256;
 };
-constexpr size_t SMEM_BYTES = Cfg<0>::SMEM > Cfg<1>::SMEM ? Cfg<0>::SMEM : Cfg<1>::SMEM;
+constexpr size_t smax(size_t a, size_t b) { return a > b ? a : b; }
+constexpr size_t SMEM_BYTES = smax(Cfg<0>::SMEM, smax(Cfg<1>::SMEM, Cfg<2>::SMEM));
+static_assert(SMEM_BYTES <= 227 * 1024, "shared memory per CTA");
 
 struct Dims {
   int num_m, num_n, num_kb;
@@ -126,56 +127,37 @@ __device__ __forceinline__ int acc_tiles_of_unit(const GemmArgs& a, int n) {
   return 1;
 }
 
-// Work layout shared by the three roles of a CTA. In the cluster modes a unit is CL consecutive
-// M tiles with one N tile (CL*mu + rank for CTA `rank` of the cluster) and units are strided
-// over clusters.
+// Work layout shared by the three roles of a CTA. In the pair modes a unit is the 2 consecutive
+// row tiles of a pair (2*mu + rank for CTA `rank`) with one column unit of NT 256-column tiles,
+// and units are strided over the resident pairs.
 template <int MODE>
 struct Sched {
-  int rank;        // CTA rank in the cluster (mode 1: 0 = leader, issues the MMAs); 0 in mode 0
+  int rank;        // CTA rank in the cluster (pair modes: 0 = leader, issues the MMAs); 0 in mode 0
   int group;       // row units per raster group
   int first, step; // unit loop: u = first; u < num_units; u += step
   int num_mu, num_nu, num_units;
 
   __device__ __forceinline__ Sched(const Dims& dm) {
     constexpr int CL = Cfg<MODE>::CL;
+    constexpr int NT = Cfg<MODE>::NT;
     rank = CL > 1 ? static_cast<int>(cluster_ctarank()) : 0;
     first = static_cast<int>(blockIdx.x) / CL;
     step = static_cast<int>(gridDim.x) / CL;
-    if (Cfg<MODE>::MC_A) {   // cluster spans column tiles
-      num_mu = dm.num_m;
-      num_nu = (dm.num_n + CL - 1) / CL;
-      group = GROUP_M;
-    } else {                 // cluster spans row tiles
-      num_mu = (dm.num_m + CL - 1) / CL;
-      num_nu = dm.num_n;
-      group = GROUP_M / CL > 0 ? GROUP_M / CL : 1;   // GROUP_M row tiles per raster group
-    }
+    num_mu = (dm.num_m + CL - 1) / CL;
+    num_nu = (dm.num_n + NT - 1) / NT;
+    group = GROUP_M / CL > 0 ? GROUP_M / CL : 1;   // GROUP_M row tiles per raster group
     num_units = num_mu * num_nu;
   }
-  // Unit u -> the row tile m and column unit n this CTA stages (always valid tiles), whether
-  // it stores its result (false for the CTAs of a cluster past the last row or, in mode 4,
-  // column tile, which only load their share of the shared operand) and the column unit n0
-  // whose accumulator count every CTA of the cluster uses: in mode 4 the CTAs of a cluster
-  // work on different column units, yet must issue the same k-blocks into the stages they
-  // share (a forward strip past the vocabulary's last tile reads zero-filled rows of W and
-  // adds nothing).
-  __device__ __forceinline__ void decode(int u, const Dims& dm, int& m, int& n, int& n0,
-                                         bool& ok) const {
+  // Unit u -> the row tile m this CTA stages (always a valid tile), the column unit n, and
+  // whether this CTA stores its result (false for the second CTA of a pair past the last row
+  // tile, which stages a copy of its leader's rows so that the pair's MMAs read valid data).
+  __device__ __forceinline__ void decode(int u, const Dims& dm, int& m, int& n, bool& ok) const {
     constexpr int CL = Cfg<MODE>::CL;
-    int mu, nu;
-    decode_unit(u, num_mu, num_nu, group, mu, nu);
-    if (Cfg<MODE>::MC_A) {
-      m = mu;
-      n0 = CL * nu;
-      n = n0 + rank;
-      ok = n < dm.num_n;
-      if (!ok) n = n0;
-    } else {
-      m = CL * mu + rank;
-      n = n0 = nu;
-      ok = m < dm.num_m;
-      if (!ok) m = CL * mu;
-    }
+    int mu;
+    decode_unit(u, num_mu, num_nu, group, mu, n);
+    m = CL * mu + rank;
+    ok = m < dm.num_m;
+    if (!ok) m = CL * mu;
   }
 };
 
@@ -231,16 +213,14 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
                              const Dims& dm, const Sched<MODE>& sc, uint8_t* sA, uint8_t* sB,
                              uint64_t* full, uint64_t* empty, volatile int* abort_flag) {
   using C = Cfg<MODE>;
-  // mode 1: only the leader's barriers count (both CTAs' bytes); modes 0, 2: every CTA's own
-  const bool leader = MODE != 1 || sc.rank == 0;
+  constexpr bool PAIR = C::PAIR;
+  constexpr int NT = C::NT;
+  // pair modes: only the leader's barriers count (both CTAs' bytes); mode 0: every CTA's own
+  const bool leader = !PAIR || sc.rank == 0;
   const bool stall = (a.inject_stall != 0) && blockIdx.x == 0;   // CTA 0 is a leader
-  constexpr int B_BOXES = static_cast<int>(C::B_LOAD_ROWS) / 64;  // MN-major B boxes loaded
-  constexpr int A_BOXES = static_cast<int>(C::A_LOAD_ROWS) / 64;  // MN-major A boxes loaded
-  const int b_col0 = (MODE == 1 || C::MC_B) ? sc.rank * static_cast<int>(C::B_LOAD_ROWS) : 0;
-  const int a_row0 = C::MC_A ? sc.rank * static_cast<int>(C::A_LOAD_ROWS) : 0;
-  // where this CTA's share of B (modes 2, 3) or A (mode 4) lands in every CTA's stage
-  const uint32_t b_off = C::MC_B ? sc.rank * C::B_LOAD_ROWS * BK * 2 : 0;
-  const uint32_t a_off = C::MC_A ? sc.rank * C::A_LOAD_ROWS * BK * 2 : 0;
+  constexpr int B_BOXES = static_cast<int>(C::B_HALF_ROWS) / 64;  // MN-major B boxes per MMA
+  // first B row (N) of this CTA's share of each 256-column MMA: the pair splits B by rows
+  const int b_row0 = PAIR ? sc.rank * static_cast<int>(C::B_HALF_ROWS) : 0;
   uint32_t stage = 0, phase = 0;
   long long issued = 0;
   bool ok = true;
@@ -248,17 +228,16 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
     int m_load, n;
     bool m_ok;
-    int n0;
-    sc.decode(u, dm, m_load, n, n0, m_ok);
-    const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
+    sc.decode(u, dm, m_load, n, m_ok);
+    const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     const int hrow = m_load * BM;   // first packed row of the tile (FWD / DZ / KL A operand)
     // The boxes of k-block kbi of accumulator tile ti: fa / fb(smem offset, map, x, y) for each
     // box of A / B this CTA loads.
     auto boxes = [&](int ti, int kbi, auto&& fa, auto&& fb) {
       if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
         const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + ti : a.vc0 / BN + n;
-        fa(0u, mapA, kbi * BK, hrow + a_row0);
-        fb(0u, mapB, kbi * BK, vt * BN + b_col0);
+        fa(0u, mapA, kbi * BK, hrow);
+        fb(0u, mapB, kbi * BK, vt * BN + b_row0);
       } else if (Dual<ROLE>::value) {
         // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
         const int nk = dm.num_kb / 2;
@@ -266,19 +245,24 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
         const int kk = second ? kbi - nk : kbi;
         const int vt = (ROLE == ROLE_FWD_KL) ? n * kFwdTilesPerStrip + ti : a.vc0 / BN + n;
         fa(0u, second ? mapA2 : mapA, kk * BK, hrow);
-        fb(0u, second ? mapB2 : mapB, kk * BK, vt * BN + b_col0);
+        fb(0u, second ? mapB2 : mapB, kk * BK, vt * BN + b_row0);
       } else if (ROLE == ROLE_DH) {
-        fa(0u, mapA, kbi * BK, m_load * BM + a_row0);
+        fa(0u, mapA, kbi * BK, m_load * BM);
 #pragma unroll
-        for (int j = 0; j < B_BOXES; ++j)
-          fb(j * BOX_MN, mapB, n * BN + b_col0 + j * 64, a.vc0 + kbi * BK);
+        for (int h = 0; h < NT; ++h)
+#pragma unroll
+          for (int j = 0; j < B_BOXES; ++j)
+            fb((h * B_BOXES + j) * BOX_MN, mapB, (n * NT + h) * BN + b_row0 + j * 64,
+               a.vc0 + kbi * BK);
       } else {  // ROLE_DW: K runs over packed rows
 #pragma unroll
-        for (int j = 0; j < A_BOXES; ++j)
-          fa(j * BOX_MN, mapA, m_load * BM + a_row0 + j * 64, kbi * BK);
+        for (int j = 0; j < BM / 64; ++j)
+          fa(j * BOX_MN, mapA, m_load * BM + j * 64, kbi * BK);
 #pragma unroll
-        for (int j = 0; j < B_BOXES; ++j)
-          fb(j * BOX_MN, mapB, n * BN + b_col0 + j * 64, kbi * BK);
+        for (int h = 0; h < NT; ++h)
+#pragma unroll
+          for (int j = 0; j < B_BOXES; ++j)
+            fb((h * B_BOXES + j) * BOX_MN, mapB, (n * NT + h) * BN + b_row0 + j * 64, kbi * BK);
       }
     };
     for (int t = 0; t < nacc && ok; ++t) {
@@ -289,25 +273,21 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
           ok = false;
           break;
         }
-        const uint32_t dA = smem_u32(sA + stage * C::A_STAGE) + a_off;
-        const uint32_t dB = smem_u32(sB + stage * C::B_STAGE) + b_off;
-        // mode 1: completion of both CTAs' copies is counted on the leader's barrier
-        const uint32_t bar = MODE == 1 ? mapa_shared(smem_u32(&full[stage]), 0)
-                                       : smem_u32(&full[stage]);
+        const uint32_t dA = smem_u32(sA + stage * C::A_STAGE);
+        const uint32_t dB = smem_u32(sB + stage * C::B_STAGE);
+        // pair modes: completion of both CTAs' copies is counted on the leader's barrier
+        const uint32_t bar = PAIR ? mapa_shared(smem_u32(&full[stage]), 0)
+                                  : smem_u32(&full[stage]);
         auto load_a = [&](uint32_t off, const CUtensorMap* map, int x, int y) {
-          if (MODE == 1) {
+          if (PAIR) {
             tma_load_2d_pair(dA + off, map, bar, x, y);
-          } else if (C::MC_A) {
-            tma_load_2d_multicast(dA + off, map, &full[stage], x, y, C::MASK);
           } else {
             tma_load_2d(dA + off, map, &full[stage], x, y);
           }
         };
         auto load_b = [&](uint32_t off, const CUtensorMap* map, int x, int y) {
-          if (MODE == 1) {
+          if (PAIR) {
             tma_load_2d_pair(dB + off, map, bar, x, y);
-          } else if (C::MC_B) {
-            tma_load_2d_multicast(dB + off, map, &full[stage], x, y, C::MASK);
           } else {
             tma_load_2d(dB + off, map, &full[stage], x, y);
           }
@@ -315,7 +295,7 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
         if (stall && issued == 0) {
           // test hook: leave stage 0 unfilled so that the MMA warp's bounded wait runs out
         } else {
-          if (leader) mbar_arrive_expect_tx(&full[stage], MODE == 1 ? 2 * C::STAGE_TX : C::STAGE_TX);
+          if (leader) mbar_arrive_expect_tx(&full[stage], PAIR ? 2 * C::STAGE_TX : C::STAGE_TX);
           boxes(t, kb, load_a, load_b);
         }
         ++issued;
@@ -326,8 +306,8 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
       }
     }
   }
-  if (ok && MODE != 0) {
-    // Cluster modes: the peer's MMAs release this CTA's stages by remote arrivals. Wait until
+  if (ok && PAIR) {
+    // Pair modes: the leader's MMAs release this CTA's stages by remote arrivals. Wait until
     // every stage has been released for the last time, so that none of them lands after this
     // CTA has left.
     for (int i = 0; i < C::STAGES; ++i) {
@@ -342,9 +322,9 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
   }
   win.leave();
   if (!ok && leader) {
-    // Aborted: let the copies already in flight land before the CTA exits (bounded). In mode 1
-    // the leader's barriers also count the peer's copies; the peer waits for the leader at the
-    // final cluster barrier.
+    // Aborted: let the copies already in flight land before the CTA exits (bounded). In the
+    // pair modes the leader's barriers also count the peer's copies; the peer waits for the
+    // leader at the final cluster barrier.
     const long long back = issued < C::STAGES ? issued : C::STAGES;
     for (long long i = 1; i <= back; ++i) {
       const long long it = issued - i;
@@ -357,15 +337,23 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
 }
 
 // ------------------------------------------------------------------------------------------
-// MMA issuer: one thread (of the leader CTA in mode 1)
+// MMA issuer: one thread (of the leader CTA in the pair modes)
 // ------------------------------------------------------------------------------------------
+// Roles and modes with one accumulator buffer: the exact-KL roles (policy and reference
+// products in the two TMEM halves) and the wide pair mode (one 512-column tile).
+template <int ROLE, int MODE>
+struct OneBuf {
+  static constexpr bool value = Dual<ROLE>::value || Cfg<MODE>::ACC_BUFS == 1;
+};
+
 template <int ROLE, int MODE>
 __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc, uint8_t* sA,
                         uint8_t* sB, uint64_t* full, uint64_t* empty, uint64_t* accf,
                         uint64_t* acce, uint64_t* drain, uint32_t tmem_base,
                         volatile int* abort_flag) {
   using C = Cfg<MODE>;
-  constexpr bool PAIR = MODE == 1;
+  constexpr bool PAIR = C::PAIR;
+  constexpr int NT = C::NT;
   if (PAIR && sc.rank != 0) return;
   constexpr bool A_MN = (ROLE == ROLE_DW);
   constexpr bool B_MN = (ROLE == ROLE_DH || ROLE == ROLE_DW);
@@ -375,9 +363,8 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
     int m_load, n;
     bool m_ok;
-    int n0;
-    sc.decode(u, dm, m_load, n, n0, m_ok);
-    const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
+    sc.decode(u, dm, m_load, n, m_ok);
+    const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     for (int t = 0; t < nacc && ok; ++t) {
       if (!mbar_wait_bounded(&acce[buf], bphase ^ 1u, abort_flag, a.hdr,
                              WHERE_GEMM_BASE + ROLE * 16 + 2)) {
@@ -404,21 +391,21 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc
         for (int k = 0; k < BK / 16; ++k) {
           const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, BOX_MN, 1024)
                                    : sdesc_sw128(a0 + k * 32, 16, 1024);
-          const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, BOX_MN, 1024)
-                                   : sdesc_sw128(b0 + k * 32, 16, 1024);
-          if (PAIR) {
-            umma_bf16_pair(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
-          } else {
-            umma_bf16(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
+#pragma unroll
+          for (int h = 0; h < NT; ++h) {   // wide pair: column halves 0-255 and 256-511
+            const uint32_t bh = b0 + h * C::B_HALF_STAGE;
+            const uint64_t bd = B_MN ? sdesc_sw128(bh + k * 2048, BOX_MN, 1024)
+                                     : sdesc_sw128(bh + k * 32, 16, 1024);
+            if (PAIR) {
+              umma_bf16_pair(dst + h * BN, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
+            } else {
+              umma_bf16(dst, ad, bd, idesc, (kr | k) != 0 ? 1u : 0u);
+            }
           }
         }
-        // frees the smem stage once these MMAs have read it: mode 1 in both CTAs of the pair;
-        // modes 2, 3 tell every CTA of the cluster, because the next multicast into this stage
-        // writes all of them
+        // frees the smem stage once these MMAs have read it (pair modes: in both CTAs)
         if (PAIR) {
           umma_commit_pair(&empty[stage], 0x3);
-        } else if (C::MC_A || C::MC_B) {
-          umma_commit_multicast(&empty[stage], C::MASK);
         } else {
           umma_commit(&empty[stage]);
         }
@@ -433,7 +420,7 @@ __device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc
       } else {
         umma_commit(&accf[buf]);
       }
-      if (Dual<ROLE>::value) {         // one buffer spanning all of TMEM
+      if (OneBuf<ROLE, MODE>::value) {  // one buffer spanning all of TMEM
         bphase ^= 1u;
       } else {
         buf ^= 1u;
@@ -464,11 +451,11 @@ __device__ __forceinline__ bool epi_wait(uint64_t* bar, uint32_t parity, volatil
   return __all_sync(0xffffffffu, ok);
 }
 
-// Tells the MMA issuer that this warp has read accumulator `bar`'s buffer; in mode 1 the
-// barrier lives in the leader CTA and counts the epilogue warps of both CTAs.
+// Tells the MMA issuer that this warp has read accumulator `bar`'s buffer; in the pair modes
+// the barrier lives in the leader CTA and counts the epilogue warps of both CTAs.
 template <int MODE>
 __device__ __forceinline__ void epi_release(uint64_t* bar, int lane, int rank) {
-  constexpr bool PAIR = MODE == 1;
+  constexpr bool PAIR = Cfg<MODE>::PAIR;
   tc_fence_before();
   __syncwarp();
   if (lane == 0) {
@@ -485,6 +472,17 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&p);
 }
 
+// Next accumulator buffer and the parity of its barriers.
+template <int ROLE, int MODE>
+__device__ __forceinline__ void advance_buf(uint32_t& buf, uint32_t& bphase) {
+  if (OneBuf<ROLE, MODE>::value) {
+    bphase ^= 1u;
+  } else {
+    buf ^= 1u;
+    if (buf == 0) bphase ^= 1u;
+  }
+}
+
 template <int ROLE, int MODE>
 __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc,
                              uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
@@ -494,12 +492,12 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
   const int r = q * 32 + lane;          // accumulator row of this thread
   const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
   const int32_t where = WHERE_GEMM_BASE + ROLE * 16 + 4;
+  constexpr int NT = Cfg<MODE>::NT;   // 256-column halves of the accumulator tile
   uint32_t buf = 0, bphase = 0;
   for (int u = sc.first; u < sc.num_units; u += sc.step) {
     int m_load, n;
-    bool m_ok;   // this CTA stores the tile (false: a cluster's CTA past the last tile)
-    int n0;
-    sc.decode(u, dm, m_load, n, n0, m_ok);
+    bool m_ok;   // this CTA stores the tile (false: a pair's second CTA past the last tile)
+    sc.decode(u, dm, m_load, n, m_ok);
 
     if (ROLE == ROLE_FWD) {
       const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
@@ -510,7 +508,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
       float rm = -INFINITY, rs = 0.f, ru = 0.f, zyv = 0.f;
       int ri = 0;
       bool found = false;
-      const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
+      const int nacc = acc_tiles_of_unit<ROLE>(a, n);
       for (int t = 0; t < nacc; ++t) {
         if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
         tc_fence_after();
@@ -581,7 +579,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
       float qm = -INFINITY, qs = 0.f;
       int ri = 0;
       bool found = false;
-      const int nacc = acc_tiles_of_unit<ROLE>(a, n0);
+      const int nacc = acc_tiles_of_unit<ROLE>(a, n);
       for (int t = 0; t < nacc; ++t) {
         if (!epi_wait(&accf[0], bphase, abort_flag, a.hdr, where)) return;
         tc_fence_after();
@@ -757,8 +755,8 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
       const long long pos = rv ? prow : 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
-      for (int c = 0; c < BN / 32; ++c) {
-        const int col = n * BN + c * 32;
+      for (int c = 0; c < NT * BN / 32; ++c) {
+        const int col = n * NT * BN + c * 32;
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
         if (!rv || col >= a.d) continue;   // columns past d (a partial last tile) hold zeros
@@ -794,8 +792,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
         }
       }
       epi_release<MODE>(&acce[buf], lane, sc.rank);
-      buf ^= 1u;
-      if (buf == 0) bphase ^= 1u;
+      advance_buf<ROLE, MODE>(buf, bphase);
 
     } else {  // ROLE_DW
       const int vrow = m_load * BM + r;
@@ -804,11 +801,11 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
       const bool empty_k = dm.num_kb == 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
-      float* dst_row = a.dW + static_cast<size_t>(a.vc0 + vrow) * a.d + n * BN;
-      for (int c = 0; c < BN / 32; ++c) {
+      float* dst_row = a.dW + static_cast<size_t>(a.vc0 + vrow) * a.d + n * NT * BN;
+      for (int c = 0; c < NT * BN / 32; ++c) {
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
-        if (!rv || n * BN + c * 32 >= a.d) continue;   // columns past d: a partial last tile
+        if (!rv || n * NT * BN + c * 32 >= a.d) continue;   // columns past d: a partial last tile
         if (empty_k) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) x[j] = 0.f;
@@ -819,8 +816,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE
           dst[j] = make_float4(x[4 * j], x[4 * j + 1], x[4 * j + 2], x[4 * j + 3]);
       }
       epi_release<MODE>(&acce[buf], lane, sc.rank);
-      buf ^= 1u;
-      if (buf == 0) bphase ^= 1u;
+      advance_buf<ROLE, MODE>(buf, bphase);
     }
   }
 }
@@ -833,7 +829,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
                                           const CUtensorMap* mapA2, const CUtensorMap* mapB2,
                                           const GemmArgs& args) {
   using C = Cfg<MODE>;
-  constexpr bool PAIR = MODE == 1;
+  constexpr bool PAIR = C::PAIR;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -852,7 +848,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], MODE >= 2 ? C::CL : 1);   // modes 2-4: every CTA's MMAs release
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
@@ -881,7 +877,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
     }
   }
   tc_fence_before();
-  if (MODE != 0) {
+  if (PAIR) {
     cluster_sync_all();  // barriers of both CTAs initialised before any cross-CTA traffic
   } else {
     __syncthreads();
@@ -904,7 +900,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   }
   __syncwarp();
   tc_fence_before();
-  if (MODE != 0) {
+  if (PAIR) {
     cluster_sync_all();  // no CTA leaves while its peer may still signal or write into it
   } else {
     __syncthreads();
@@ -927,32 +923,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   gemm_body<ROLE, 0>(&mapA, &mapB, &mapA2, &mapB2, args);
 }
 
-template <int ROLE>
+// MODE 1 (256 x 256 tiles) or 2 (256 x 512 tiles) on CTA pairs.
+template <int ROLE, int MODE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_pair(const __grid_constant__ CUtensorMap mapA,
                  const __grid_constant__ CUtensorMap mapB, const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, 1>(&mapA, &mapB, &mapA, &mapB, args);
+  gemm_body<ROLE, MODE>(&mapA, &mapB, &mapA, &mapB, args);
 }
 
-template <int ROLE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-    tc_gemm_mc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-               const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, 2>(&mapA, &mapB, &mapA, &mapB, args);
-}
-
-template <int ROLE>
-__global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-    tc_gemm_mc4(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-                const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, 3>(&mapA, &mapB, &mapA, &mapB, args);
-}
-
-template <int ROLE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-    tc_gemm_mca(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-                const __grid_constant__ GemmArgs args) {
-  gemm_body<ROLE, 4>(&mapA, &mapB, &mapA, &mapB, args);
+template <class Kernel, class... Args>
+cudaError_t launch_with_smem(Kernel kernel, size_t smem, int grid, cudaStream_t st,
+                             Args&&... args) {
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  kernel<<<grid, NUM_THREADS, smem, st>>>(args...);
+  return cudaGetLastError();
 }
 
 template <int ROLE>
@@ -960,64 +946,26 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
                         int grid, int mode, cudaStream_t st, const CUtensorMap& mapA2,
                         const CUtensorMap& mapB2) {
   if constexpr (!Dual<ROLE>::value) {       // exact-KL roles: single-CTA tiles only
-    if (mode == 1) {
-      const size_t smem = Cfg<1>::SMEM;
-      cudaError_t e = cudaFuncSetAttribute(tc_gemm_pair<ROLE>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           static_cast<int>(smem));
-      if (e != cudaSuccess) return e;
-      tc_gemm_pair<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
-      return cudaGetLastError();
-    }
-    if (mode == 2) {
-      const size_t smem = Cfg<2>::SMEM;
-      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mc<ROLE>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           static_cast<int>(smem));
-      if (e != cudaSuccess) return e;
-      tc_gemm_mc<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
-      return cudaGetLastError();
-    }
-    if (mode == 3) {
-      const size_t smem = Cfg<3>::SMEM;
-      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mc4<ROLE>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           static_cast<int>(smem));
-      if (e != cudaSuccess) return e;
-      tc_gemm_mc4<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
-      return cudaGetLastError();
-    }
-    if (mode == 4) {
-      const size_t smem = Cfg<4>::SMEM;
-      cudaError_t e = cudaFuncSetAttribute(tc_gemm_mca<ROLE>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           static_cast<int>(smem));
-      if (e != cudaSuccess) return e;
-      tc_gemm_mca<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, args);
-      return cudaGetLastError();
+    if (mode == 1)
+      return launch_with_smem(tc_gemm_pair<ROLE, 1>, Cfg<1>::SMEM, grid, st, mapA, mapB, args);
+    if constexpr (ROLE == ROLE_DH || ROLE == ROLE_DW) {   // wide pair: the long-K roles only
+      if (mode == 2)
+        return launch_with_smem(tc_gemm_pair<ROLE, 2>, Cfg<2>::SMEM, grid, st, mapA, mapB, args);
     }
   }
-  {
-    const size_t smem = Cfg<0>::SMEM;
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm<ROLE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    tc_gemm<ROLE><<<grid, NUM_THREADS, smem, st>>>(mapA, mapB, mapA2, mapB2, args);
-  }
-  return cudaGetLastError();
+  if (mode != 0) return cudaErrorInvalidValue;
+  return launch_with_smem(tc_gemm<ROLE>, Cfg<0>::SMEM, grid, st, mapA, mapB, mapA2, mapB2, args);
 }
 
 }  // namespace
 
 size_t gemm_smem_bytes() { return SMEM_BYTES; }
 
-int gemm_cluster_size(int tile_mode) { return tile_mode == 3 ? 4 : (tile_mode != 0 ? 2 : 1); }
+int gemm_cluster_size(int tile_mode) { return tile_mode != 0 ? 2 : 1; }
 
-int gemm_b_box_rows(int tile_mode) {
-  return (tile_mode == 0 || tile_mode == 4) ? BN : BN / 2 / (tile_mode == 3 ? 2 : 1);
-}
+int gemm_col_tiles_per_unit(int tile_mode) { return tile_mode == 2 ? 2 : 1; }
 
-int gemm_a_box_rows(int tile_mode) { return tile_mode == 4 ? BM / 2 : BM; }
+int gemm_b_box_rows(int tile_mode) { return tile_mode == 0 ? BN : BN / 2; }
 
 namespace {
 template <typename Kernel>
@@ -1039,7 +987,7 @@ int query_active_clusters(Kernel kernel, size_t smem, int cl) {
 }
 
 constexpr int kMaxDevices = 64;
-std::atomic<int> g_active_clusters[kMaxDevices][5];   // 0 = not queried yet
+std::atomic<int> g_active_clusters[kMaxDevices][3];   // 0 = not queried yet
 }  // namespace
 
 int gemm_max_clusters(int tile_mode) {
@@ -1049,25 +997,23 @@ int gemm_max_clusters(int tile_mode) {
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return 1;
   int cap = sms / cl > 0 ? sms / cl : 1;
-  if (cl == 1 || dev < 0 || dev >= kMaxDevices || tile_mode < 0 || tile_mode > 4) return cap;
+  if (cl == 1 || dev < 0 || dev >= kMaxDevices || tile_mode < 0 || tile_mode > 2) return cap;
   int known = g_active_clusters[dev][tile_mode].load();
   if (known == 0) {
     int n = 0;
-    if (tile_mode == 1) n = query_active_clusters(tc_gemm_pair<ROLE_FWD>, Cfg<1>::SMEM, cl);
-    if (tile_mode == 2) n = query_active_clusters(tc_gemm_mc<ROLE_FWD>, Cfg<2>::SMEM, cl);
-    if (tile_mode == 3) n = query_active_clusters(tc_gemm_mc4<ROLE_FWD>, Cfg<3>::SMEM, cl);
-    if (tile_mode == 4) n = query_active_clusters(tc_gemm_mca<ROLE_FWD>, Cfg<4>::SMEM, cl);
+    if (tile_mode == 1) n = query_active_clusters(tc_gemm_pair<ROLE_FWD, 1>, Cfg<1>::SMEM, cl);
+    if (tile_mode == 2) n = query_active_clusters(tc_gemm_pair<ROLE_DW, 2>, Cfg<2>::SMEM, cl);
     known = n > 0 ? n : cap;   // a failed query falls back to one cluster per `cl` SMs
     g_active_clusters[dev][tile_mode].store(known);
   }
   return known < cap ? known : cap;
 }
 
-int gemm_grid(long long row_units, long long col_units, int tile_mode) {
+int gemm_grid(long long row_tiles, long long col_tiles, int tile_mode) {
   const long long cl = gemm_cluster_size(tile_mode);
+  const long long nt = gemm_col_tiles_per_unit(tile_mode);
   const long long cap = gemm_max_clusters(tile_mode);
-  const long long units = tile_mode == 4 ? row_units * ((col_units + cl - 1) / cl)
-                                         : ((row_units + cl - 1) / cl) * col_units;
+  const long long units = ((row_tiles + cl - 1) / cl) * ((col_tiles + nt - 1) / nt);
   return static_cast<int>(cl * (units < cap ? (units > 0 ? units : 1) : cap));
 }
 

@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <functional>
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -71,6 +72,13 @@ struct GemmArgs {
 // Fills the progress-window fields of `a` from the process-wide setting (grpo_set_gemm_window).
 void gemm_window_config(GemmArgs& a);
 
+// Kernel accounting of the C ABI (grpo_timing_*): runs `launch` (which enqueues one kernel of
+// kind `kernel_id`, a GRPO_K_* value, on `st`), counts it and, with timing on, brackets it with
+// events on `st`. Returns GRPO_OK or GRPO_ERR_CUDA (GRPO_ERR_INVALID_ARG for a bad id).
+int counted_launch(int kernel_id, cudaStream_t st, const std::function<cudaError_t()>& launch);
+// Current value of the grpo_debug_inject_stall test hook (nonzero = on).
+int debug_inject_stall();
+
 // Launches (all asynchronous on `st`; return the cudaError_t of the launch).
 cudaError_t launch_mask_scan(const uint8_t* mask, int S, int T, int32_t* counts,
                              cudaStream_t st);
@@ -132,28 +140,29 @@ cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
                           const uint8_t* mask, const float* lse, const float* g, int S, int T,
                           int d, int V, float* dW, cudaStream_t st);
 
-// Tensor-core tile mode (0 single CTA, 1 CTA pair with cta_group::2, 2 / 3 single-CTA MMAs
-// sharing B by TMA multicast in a 2- / 4-CTA cluster, 4 sharing A by TMA multicast in a 2-CTA
-// cluster) that GEMM role `role` (ROLE_*) runs in,
-// (the process-wide mode chosen through grpo_set_tile_mode).
+// Tensor-core tile mode that GEMM role `role` (ROLE_*) runs in (the process-wide choice made
+// through grpo_set_tile_mode / grpo_set_role_tile_mode): 0 single CTA, 128 x 256 tiles
+// (cta_group::1); 1 CTA pair, 256 x 256 tiles (cta_group::2); 2 CTA pair, 256 x 512 tiles (DH
+// and DW only).
 int gemm_role_tile_mode(int role);
 
 // tcgen05 GEMM launches. `grid` = persistent CTAs.
 size_t gemm_smem_bytes();
-// CTAs per cluster of a tile mode (1, 2 or 4) and the rows of the K-major B box each CTA loads.
+// CTAs per cluster of a tile mode (1 or 2), 256-column tiles per work unit (1, or 2 in mode 2)
+// and the rows of the K-major B box each CTA loads (256, or 128 in the pair modes: the pair
+// splits B by rows). A boxes are always 128 rows (K-major) or 64 x 64 (MN-major).
 int gemm_cluster_size(int tile_mode);
+int gemm_col_tiles_per_unit(int tile_mode);
 int gemm_b_box_rows(int tile_mode);
-// Rows of the K-major A box each CTA loads (64 in mode 4, where two CTAs share A; else 128).
-int gemm_a_box_rows(int tile_mode);
 // Clusters of a tile mode that can be resident at once (cudaOccupancyMaxActiveClusters, cached
 // per device), at most one per `cluster size` SMs.
 int gemm_max_clusters(int tile_mode);
-// Persistent grid for `row_units` x `col_units` output tiles of 128 rows: one CTA per SM, or in
-// the cluster modes as many clusters as can be resident, each taking `cluster size`
-// consecutive row tiles per unit; never more CTAs than units need.
-int gemm_grid(long long row_units, long long col_units, int tile_mode);
-// tile_mode 1, 2, 3: cluster kernels; `grid` must be a multiple of the cluster size and the
-// K-major B map's box gemm_b_box_rows(tile_mode) rows (each CTA loads its share of B).
+// Persistent grid for `row_tiles` x `col_tiles` output tiles of 128 x 256: one CTA per SM, or in
+// the pair modes as many pairs as can be resident, each taking 2 consecutive row tiles (and, in
+// mode 2, 2 consecutive column tiles) per unit; never more CTAs than units need.
+int gemm_grid(long long row_tiles, long long col_tiles, int tile_mode);
+// tile_mode 1, 2: pair kernels; `grid` must be even and the K-major B map's box
+// gemm_b_box_rows(tile_mode) rows. Mode 2 is accepted for ROLE_DH and ROLE_DW only.
 // mapA2 / mapB2 (H_ref, W_ref) are read by the KL roles only (single-CTA tiles).
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const GemmArgs& args, int grid, int tile_mode, cudaStream_t st,

@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libgrpo_gb300.so")
 HEADER_PATH = os.path.join(os.path.dirname(_HERE), "include", "grpo.h")
 
 GRPO_F32, GRPO_BF16 = 0, 1
+STATIC_SCRATCH_BYTES = 64 << 20      # GRPO_STATIC_SCRATCH_BYTES of include/grpo.h
 STD_MODES = {"unbiased": 0, "population": 1}
 AGG_MODES = {"seq_mean": 0, "token_mean": 1}
 STATUS_NAMES = {0: "GRPO_OK", -1: "GRPO_ERR_INVALID_ARG", -2: "GRPO_ERR_UNSUPPORTED",
@@ -477,14 +478,13 @@ def grpo_set_cta_pair(on: bool):
 
 
 TILE_DEFAULT = -1
-TILE_SINGLE, TILE_CTA_PAIR, TILE_MULTICAST, TILE_MULTICAST4, TILE_MULTICAST_A = 0, 1, 2, 3, 4
+TILE_SINGLE, TILE_CTA_PAIR, TILE_CTA_PAIR_WIDE = 0, 1, 2
 ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW = 0, 1, 2, 3
 
 
 def grpo_set_tile_mode(mode: int):
-    """Every GEMM role in one mode: 0 single-CTA tiles, 1 CTA pairs (cta_group::2), 2 / 3 B
-    tile shared by TMA multicast in clusters of 2 / 4 CTAs, 4 A tile shared by TMA multicast in
-    2-CTA clusters; -1 (TILE_DEFAULT) restores each role's default."""
+    """Every GEMM role in one mode: 0 single-CTA 128 x 256 tiles, 1 CTA-pair 256 x 256 tiles
+    (cta_group::2); -1 (TILE_DEFAULT) restores each role's default."""
     _check(_lib().grpo_set_tile_mode(int(mode)), "grpo_set_tile_mode")
 
 
@@ -494,8 +494,8 @@ def grpo_get_tile_mode() -> int:
 
 
 def grpo_set_role_tile_mode(role: int, mode: int):
-    """Tile mode of one GEMM role (ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW); -1 restores the
-    role's default."""
+    """Tile mode of one GEMM role (ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW): 0, 1, or for ROLE_DH and
+    ROLE_DW also 2 (CTA-pair 256 x 512 tiles); -1 restores the role's default."""
     _check(_lib().grpo_set_role_tile_mode(int(role), int(mode)), "grpo_set_role_tile_mode")
 
 

@@ -24,6 +24,22 @@ def test_reference_arm_prints_contract_line():
     assert line["config"]["workload"] == "g8_t1k_d2048_v32k"
 
 
+def test_gpus_flag_launches_one_process_per_gpu():
+    """`bench.py --gpus 2` without a torch.distributed environment re-launches itself under
+    torch.distributed.run with two ranks (127.0.0.1 rendezvous); for the reference arm rank 0
+    alone prints the line, with n_gpus = 2, and the other rank exits 0."""
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2",
+           "--steps", "1", "--warmup", "0", "--config", "g8_t1k_d2048_v32k", "--ref-tokens", "2",
+           "--master-port", "29541"]
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK")}
+    out = subprocess.run(cmd, capture_output=True, text=True, timeout=600, cwd=ROOT, env=env)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [json.loads(x) for x in out.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1
+    assert lines[0]["n_gpus"] == 2 and lines[0]["impl"] == "reference"
+    assert lines[0]["cpu_baseline"]["cores"] >= 1
+
+
 def test_traffic_figure_is_keyed_to_kernel_source_and_tile_mode(tmp_path, monkeypatch):
     """The roofline's `traffic` comes from a committed ncu summary only if that summary was taken
     on the current GEMM source in the tile mode the kernel runs in now (a summary without a

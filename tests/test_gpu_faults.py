@@ -78,18 +78,14 @@ def test_bad_group_offsets_set_status():
     assert np.isfinite(a.cpu().numpy()).all()
 
 
-@pytest.mark.parametrize("mode", [1, 2, 3, 4],
-                         ids=["cta_pair", "multicast2", "multicast4", "multicast_a"])
-def test_stalled_pipeline_times_out_in_cluster_tile_modes(mode):
-    """The same injected stall with 2-CTA clusters. Mode 1 (CTA pairs): the leader's MMA wait
-    runs out. Modes 2-4 (B or A multicast): CTA 0 loads neither its own operand nor its share of
-    the shared one, so the MMA waits of every CTA in its cluster run out. Every CTA leaves through its bounded waits and the final
-    cluster barrier, and the next call is correct."""
+def test_stalled_pipeline_times_out_in_cta_pair_tiles():
+    """The same injected stall with CTA pairs (mode 1, every GEMM role): the leader's MMA wait
+    runs out, its peer's producer wait runs out after it, both leave through their bounded waits
+    and the final cluster barrier, and the next call is correct."""
     b, (H, W, tok, mask) = _small()
     S, T, d = H.shape
     ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
-    prev = G.grpo_get_tile_mode()
-    G.grpo_set_tile_mode(mode)
+    G.grpo_set_tile_mode(G.TILE_CTA_PAIR)
     try:
         good = {k: v.clone() for k, v in G.grpo_score_fwd(H, W, tok, mask, ws).items()}
         assert G.grpo_last_device_error(ws)[0] == 0
@@ -106,4 +102,41 @@ def test_stalled_pipeline_times_out_in_cluster_tile_modes(mode):
         for k in ("logp", "lse", "entropy", "argmax"):
             assert torch.equal(again[k], good[k]), k
     finally:
-        G.grpo_set_tile_mode(prev)
+        G.grpo_set_tile_mode(G.TILE_DEFAULT)
+
+
+def test_stalled_backward_times_out_in_wide_pair_tiles():
+    """The injected stall in a backward whose dH and dW GEMMs run 256 x 512 CTA-pair tiles (the
+    default): every GEMM of the call (dz recompute, dH, dW) gives up through its bounded waits and
+    records GRPO_ERR_TIMEOUT, and the next backward on the same context gives bitwise the
+    gradients of one made before the stall."""
+    b, (H, W, tok, mask) = _small()
+    S, T, d = H.shape
+    ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
+    G.grpo_set_tile_mode(G.TILE_DEFAULT)
+    assert [G.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 0, 2, 2]
+    dev = H.device
+    adv = G.group_advantages(b.rewards.to(dev), b.group_offsets.to(dev), ws)
+    f = G.grpo_score_fwd(H, W, tok, mask, ws)
+    old = (f["logp"] + b.noise_old.to(dev)).contiguous()
+    ref = (f["logp"] + b.noise_ref.to(dev)).contiguous()
+
+    def backward():
+        r = G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old, ref, adv,
+                            f["valid_count"], ws)
+        return {k: v.clone() for k, v in r.items()}
+
+    good = backward()
+    assert G.grpo_last_device_error(ws)[0] == 0
+    G.grpo_debug_inject_stall(True)
+    try:
+        backward()
+        st, where = G.grpo_last_device_error(ws)
+    finally:
+        G.grpo_debug_inject_stall(False)
+    assert st == TIMEOUT, (st, where)
+    again = backward()
+    torch.cuda.synchronize()
+    assert G.grpo_last_device_error(ws)[0] == 0
+    for k in ("loss", "dH", "dW"):
+        assert torch.equal(again[k], good[k]), k
