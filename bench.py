@@ -259,6 +259,46 @@ def cpu_baseline(w, n_tokens, steps=1, warmup=0):
                       f"threads; mean of {len(times)} run(s)"}
 
 
+def run_e2e(step, dev_args, stream, device, e2e_steps, ws_n):
+    """Times `e2e_steps` steps whose inputs come from pinned host memory (double-buffered copies
+    on a second stream) and whose loss is read back; returns (seconds, host->device bytes/step)."""
+    names = ("H", "W", "tokens", "mask", "rewards", "go", "old", "ref")
+    host = {k: v.cpu().pin_memory() for k, v in zip(names, dev_args)}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    sets = [dev_args, tuple(torch.empty_like(v) for v in dev_args)]
+    copy_stream = torch.cuda.Stream(device)
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    used = [torch.cuda.Event(), torch.cuda.Event()]
+    loss_host = torch.empty(e2e_steps, dtype=torch.float32).pin_memory()
+
+    def upload(j):
+        with torch.cuda.stream(copy_stream):
+            if j >= 2:
+                copy_stream.wait_event(used[j % 2])     # step j-2 is done with this set
+            for k, dst in zip(names, sets[j % 2]):
+                dst.copy_(host[k], non_blocking=True)
+            copied[j % 2].record(copy_stream)
+
+    torch.cuda.synchronize()
+    barrier(ws_n)
+    t0 = time.perf_counter()
+    upload(0)
+    for j in range(e2e_steps):
+        if j + 1 < e2e_steps:
+            upload(j + 1)
+        stream.wait_event(copied[j % 2])
+        r = step(*sets[j % 2])
+        used[j % 2].record(stream)
+        loss_host[j:j + 1].copy_(r["loss"], non_blocking=True)
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    barrier(ws_n)
+    e2e_s = dist_max(e2e_s, ws_n, device)
+    if not bool(torch.isfinite(loss_host).all()):
+        raise RuntimeError("non-finite loss in the end-to-end steps")
+    return e2e_s, h2d
+
+
 # ---------------------------------------------------------------------------------------------
 def run_gpu(args):
     ws_n, rank, local = dist_env()
@@ -278,6 +318,8 @@ def run_gpu(args):
     G.grpo_set_gemm_window(win[0], win[1])
     w = apply_scale(WORKLOADS[args.config], args.scale)
     w = w.scaled(seed=w.seed + 1000 * rank)        # each rank scores its own groups
+    if args.beta is not None:
+        w = w.scaled(beta=args.beta)
     t_gen = time.time()
     b = make_batch_torch(w, device=str(device))
     S, T, d, V = w.S, w.T, w.d, w.V
@@ -313,6 +355,8 @@ def run_gpu(args):
                                        ws, out=bwd_out)
         G.group_advantages(rewards, go, ws, adv_out=adv)
         f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
+        if w.beta == 0.0:          # no KL term: the reference log-probs are not read
+            ref_ = None
         return G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_, ref_, adv,
                                f["valid_count"], ws, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
                                out=bwd_out)
@@ -366,46 +410,15 @@ def run_gpu(args):
     # Every step's inputs are copied from pinned host memory and its loss read back inside the
     # timed region. Inputs are double-buffered: step j+1's copies run on a second stream while
     # step j computes (GB300's C2C link moves the 6.9 GB in a few percent of a step).
-    names = ("H", "W", "tokens", "mask", "rewards", "go", "old", "ref")
-    host = {k: v.cpu().pin_memory() for k, v in zip(names, dev_args)}
-    h2d = sum(v.numel() * v.element_size() for v in host.values())
-    e2e_steps = max(1, args.e2e_steps)
-    sets = [dev_args, tuple(torch.empty_like(v) for v in dev_args)]
-    copy_stream = torch.cuda.Stream(device)
-    copied = [torch.cuda.Event(), torch.cuda.Event()]
-    used = [torch.cuda.Event(), torch.cuda.Event()]
-    loss_host = torch.empty(e2e_steps, dtype=torch.float32).pin_memory()
-
-    def upload(j):
-        with torch.cuda.stream(copy_stream):
-            if j >= 2:
-                copy_stream.wait_event(used[j % 2])     # step j-2 is done with this set
-            for k, dst in zip(names, sets[j % 2]):
-                dst.copy_(host[k], non_blocking=True)
-            copied[j % 2].record(copy_stream)
-
-    torch.cuda.synchronize()
-    barrier(ws_n)
-    t0 = time.perf_counter()
-    upload(0)
-    for j in range(e2e_steps):
-        if j + 1 < e2e_steps:
-            upload(j + 1)
-        stream.wait_event(copied[j % 2])
-        r = step(*sets[j % 2])
-        used[j % 2].record(stream)
-        loss_host[j:j + 1].copy_(r["loss"], non_blocking=True)
-    torch.cuda.synchronize()
-    e2e_s = time.perf_counter() - t0
-    barrier(ws_n)
-    e2e_s = dist_max(e2e_s, ws_n, device)
-    if not bool(torch.isfinite(loss_host).all()):
-        raise RuntimeError("non-finite loss in the end-to-end steps")
-    del sets
+    # --e2e-steps 0 skips this part (profiling captures: no second copy of the inputs).
+    e2e_steps = args.e2e_steps
+    e2e_s = h2d = None
+    if e2e_steps > 0:
+        e2e_s, h2d = run_e2e(step, dev_args, stream, device, e2e_steps, ws_n)
 
     total_tokens = dist_sum(float(N_v), ws_n, device)
     value = total_tokens * args.steps / (ms_max / 1e3)
-    e2e_value = total_tokens * e2e_steps / e2e_s
+    e2e_value = total_tokens * e2e_steps / e2e_s if e2e_steps > 0 else None
     pk = peaks()
     step_ms = ms_max / args.steps
     # algorithmic flop per step: 6 N d V (fwd, dH, dW); the exact-KL path adds the reference
@@ -451,7 +464,7 @@ def run_gpu(args):
         "ms_per_step": round(step_ms, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "prompts": w.prompts, "G": list(w.group_sizes), "T": T,
-                   "d": d, "V": V, "scored_tokens_per_rank": N_v,
+                   "d": d, "V": V, "eps": w.eps, "beta": w.beta, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
                    "tiles": tiles_desc(G),
                    "gemm_window": ("off" if win[0] == 0 else
@@ -467,10 +480,11 @@ def run_gpu(args):
         "roofline": roof,
         "kernels": per_kernel,
         "gpu_launches": launches,
-        "e2e": {"value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": 4, "steps": e2e_steps,
-                "copies": "pinned host -> device every step; step j+1's inputs copied on a "
-                          "second stream while step j computes"},
+        "e2e": None if e2e_value is None else {
+            "value": round(e2e_value, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": 4, "steps": e2e_steps,
+            "copies": "pinned host -> device every step; step j+1's inputs copied on a "
+                      "second stream while step j computes"},
         "clocks": clk.summary(),
         "setup_s": round(gen_s, 1),
     }
@@ -492,7 +506,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--vocab-chunk", type=int, default=0)
+    ap.add_argument("--vocab-chunk", type=int, default=0,
+                    help="vocabulary columns of dz kept at once (0 = whole vocabulary)")
+    ap.add_argument("--beta", type=float, default=None,
+                    help="KL coefficient (default: the workload's); 0 = no KL term, reference "
+                         "log-probs not read")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-tokens", type=int, default=32)
     ap.add_argument("--ref-tokens", type=int, default=16)

@@ -213,8 +213,34 @@ __global__ void k_group_adv(const float* __restrict__ r, const int32_t* __restri
 
 // ------------------------------------------------------------------------------------------
 // Merge of per-strip statistics (max m, sum s = sum e^{z-m}, u = sum e^{z-m} z, argmax) into
-// lse, logp, entropy, argmax; one thread per position.
+// lse, logp, entropy, argmax; one thread per position, one pass over the strips in vocabulary
+// order with the running sums rescaled whenever the running maximum rises (so ties keep the
+// lowest index).
 // ------------------------------------------------------------------------------------------
+struct StripMerge {
+  float M = -INFINITY, S = 0.f, U = 0.f;
+  int idx = 0;
+  // Adds strip statistics p = (m, s, u, argmax bits); returns the factor e^{m - M} that scales
+  // quantities summed with e^{z - m} weights into the running maximum's frame.
+  __device__ __forceinline__ float add(const float4 p) {
+    if (p.x > M) {
+      const float r = ex2_approx((M - p.x) * kLog2e);   // 0 on the first strip (M = -inf)
+      S = fmaf(S, r, p.y);
+      U = fmaf(U, r, p.z);
+      M = p.x;
+      idx = __float_as_int(p.w);
+      rescale = r;
+      return 1.f;
+    }
+    const float sc = ex2_approx((p.x - M) * kLog2e);
+    S = fmaf(p.y, sc, S);
+    U = fmaf(p.z, sc, U);
+    rescale = 1.f;
+    return sc;
+  }
+  float rescale = 1.f;   // factor the running sums were multiplied by in the last add()
+};
+
 __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_cap,
                             int num_strips, const float* __restrict__ zy,
                             const int32_t* __restrict__ pos_row,
@@ -232,22 +258,10 @@ __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_
     return;
   }
   const long long row = pos_row[pos];   // packed row of this scored position
-  float M = -INFINITY;
-  int idx = 0;
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    if (p.x > M) {
-      M = p.x;
-      idx = __float_as_int(p.w);
-    }
-  }
-  float Ssum = 0.f, U = 0.f;
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    const float sc = ex2_approx((p.x - M) * kLog2e);
-    Ssum = fmaf(p.y, sc, Ssum);
-    U = fmaf(p.z, sc, U);
-  }
+  StripMerge mg;
+  for (int j = 0; j < num_strips; ++j) mg.add(partials[static_cast<long long>(j) * rows_cap + row]);
+  const float M = mg.M, Ssum = mg.S, U = mg.U;
+  const int idx = mg.idx;
   const float lse = M + logf(Ssum);
   const int y = tokens[pos];
   float lp;
@@ -287,27 +301,23 @@ __global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
     return;
   }
   const long long row = pos_row[pos];   // packed row of this scored position
-  float M = -INFINITY, Mr = -INFINITY;
-  int idx = 0;
+  StripMerge mg;                        // policy: (m, s, u, argmax)
+  float C = 0.f;                        // sum e^{z-M} z_ref in the policy's frame
+  float Mr = -INFINITY, Sr = 0.f;       // reference: running max and sum e^{z_ref - Mr}
   for (int j = 0; j < num_strips; ++j) {
     const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
     const float4 q = partials2[static_cast<long long>(j) * rows_cap + row];
-    if (p.x > M) {
-      M = p.x;
-      idx = __float_as_int(p.w);
+    const float sc = mg.add(p);
+    C = fmaf(C, mg.rescale, q.x * sc);
+    if (q.y > Mr) {
+      Sr = fmaf(Sr, ex2_approx((Mr - q.y) * kLog2e), q.z);
+      Mr = q.y;
+    } else {
+      Sr = fmaf(q.z, ex2_approx((q.y - Mr) * kLog2e), Sr);
     }
-    Mr = fmaxf(Mr, q.y);
   }
-  float Ssum = 0.f, U = 0.f, C = 0.f, Sr = 0.f;
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    const float4 q = partials2[static_cast<long long>(j) * rows_cap + row];
-    const float sc = ex2_approx((p.x - M) * kLog2e);
-    Ssum = fmaf(p.y, sc, Ssum);
-    U = fmaf(p.z, sc, U);
-    C = fmaf(q.x, sc, C);
-    Sr = fmaf(q.z, ex2_approx((q.y - Mr) * kLog2e), Sr);
-  }
+  const float M = mg.M, Ssum = mg.S, U = mg.U;
+  const int idx = mg.idx;
   const float lse = M + logf(Ssum);
   const float lser = Mr + logf(Sr);
   const int y = tokens[pos];
@@ -456,23 +466,9 @@ __global__ void k_shard_stats(const float4* __restrict__ partials, long long row
     return;
   }
   const long long row = pos_row[pos];   // packed row of this scored position
-  float M = -INFINITY;
-  int idx = 0;
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    if (p.x > M) {
-      M = p.x;
-      idx = __float_as_int(p.w);
-    }
-  }
-  float Ssum = 0.f, U = 0.f;
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    const float sc = ex2_approx((p.x - M) * kLog2e);
-    Ssum = fmaf(p.y, sc, Ssum);
-    U = fmaf(p.z, sc, U);
-  }
-  stats[pos] = make_float4(M, Ssum, U, __int_as_float(idx + v_offset));
+  StripMerge mg;
+  for (int j = 0; j < num_strips; ++j) mg.add(partials[static_cast<long long>(j) * rows_cap + row]);
+  stats[pos] = make_float4(mg.M, mg.S, mg.U, __int_as_float(mg.idx + v_offset));
   const int yl = tokens[pos] - v_offset;
   zy_out[pos] = (yl >= 0 && yl < V_shard) ? zy_ws[pos] : -INFINITY;
 }
