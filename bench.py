@@ -468,7 +468,8 @@ def run_gpu(args):
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
                    "tiles": tiles_desc(G),
                    "gemm_window": ("off" if win[0] == 0 else
-                                   f"{win[0]} k-blocks, lag {win[1]} checkpoints"),
+                                   f"{win[0]} k-blocks, lag {win[1]} checkpoints" if win[0] > 0
+                                   else f"every {-win[0]} work unit(s), lag {win[1]}"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
                        b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
                    "parallelism": f"dp{ws_n} (independent groups per GPU)",
@@ -527,7 +528,8 @@ def main():
                          "(-1 = that GEMM's default; 2 = " + TILE_MODES[2] + ", dH and dW only)")
     ap.add_argument("--gemm-window", default="0,0",
                     help="GEMM progress window CHECK,LAG: producers stay within LAG checkpoints of "
-                         "CHECK k-blocks of the launch's average ('0,0' = off)")
+                         "the launch's average; checkpoints every CHECK k-blocks, or at every "
+                         "-CHECK-th work unit for CHECK < 0 (write --gemm-window=-1,1); '0,0' = off")
     ap.add_argument("--graph", action="store_true",
                     help="capture one step in a CUDA graph and time its replays (per-kernel "
                          "timing and launch counts then come from the capture, not the replays)")

@@ -101,7 +101,7 @@ int grpo_score_fwd(const void* H, const void* W, int32_t dtype, const int32_t* t
  * Arguments, outputs and results are those of grpo_score_fwd, except:
  *  - the scratch is a GRPO_STATIC_SCRATCH_BYTES (64 MiB) __device__ array inside the library,
  *    held on every GPU that loads the library until the process exits. A batch whose scratch
- *    (for bf16 about R * (16 * ceil(V/2048) + 2 * d + 4) + 8 * S*T bytes, R = S*T rounded up to
+ *    (for bf16 about R * (16 * ceil(V/256) + 2 * d + 4) + 8 * S*T bytes, R = S*T rounded up to
  *    a multiple of 128) does not fit returns GRPO_ERR_WORKSPACE before anything is enqueued;
  *  - it allocates nothing and calls no allocating routine;
  *  - the first call made with a given device current looks up the array's device address
@@ -295,13 +295,15 @@ int grpo_set_cta_pair(int32_t on);
 int grpo_set_role_tile_mode(int32_t role, int32_t mode);
 int grpo_get_role_tile_mode(int32_t role);
 
-/* Progress window of the tensor-core GEMMs, process-wide, for launches made afterwards. Every
- * `check_kblocks` k-blocks of 64 the TMA producer of each CTA waits (at most 0.5 ms) until the
- * CTAs of the launch are on average within `lag` such checkpoints of it, so that CTAs reading the
- * same operand tiles read them close enough in time to hit L2 (long-K GEMMs otherwise drift apart
- * and re-read their operands from HBM). Results do not depend on it. check_kblocks == 0 turns it
- * off (the default: on a power-capped GB300 the waits cost more than the L2 hits gain). Returns GRPO_ERR_INVALID_ARG for negative values or for
- * check_kblocks > 0 with lag == 0. */
+/* Progress window of the tensor-core GEMMs, process-wide, for launches made afterwards. At every
+ * checkpoint the TMA producer of each CTA waits (at most 0.5 ms) until the CTAs of the launch are
+ * on average within `lag` checkpoints of it, so that CTAs reading the same operand tiles read
+ * them close enough in time to hit L2 (long-K GEMMs otherwise drift apart and re-read their
+ * operands from HBM). Checkpoints fall every `check_kblocks` k-blocks of 64 (check_kblocks > 0)
+ * or, for check_kblocks < 0, at the start of every (-check_kblocks)-th work unit (an output
+ * tile or strip): with lag 1 a barrier between the waves of units. Results do not depend on it.
+ * check_kblocks == 0 turns it off (the default). Returns GRPO_ERR_INVALID_ARG for a negative lag
+ * or for check_kblocks != 0 with lag == 0. */
 int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag);
 
 #ifdef __cplusplus

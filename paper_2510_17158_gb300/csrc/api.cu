@@ -795,9 +795,9 @@ int grpo_get_role_tile_mode(int32_t role) {
 }
 
 int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag) {
-  if (check_kblocks < 0 || lag < 0 || (check_kblocks > 0 && lag == 0)) return GRPO_ERR_INVALID_ARG;
+  if (lag < 0 || (check_kblocks != 0 && lag == 0)) return GRPO_ERR_INVALID_ARG;
   g_win_check.store(check_kblocks);
-  g_win_lag.store(check_kblocks > 0 ? lag : 0);
+  g_win_lag.store(check_kblocks != 0 ? lag : 0);
   return GRPO_OK;
 }
 

@@ -1,8 +1,8 @@
 // Persistent, warp-specialised tcgen05 GEMM for the four LM-head contractions of the GRPO path.
 //
 //   role FWD : z = H W^T per 128-token x 256-vocab tile (K = d), reduced on chip to the
-//              running max / sum e^{z-m} / sum e^{z-m} z / argmax / target logit of each token
-//              over a strip of 8 vocabulary tiles (Eq. 1's log pi: log-softmax at the sampled
+//              max / sum e^{z-m} / sum e^{z-m} z / argmax / target logit of each token over the
+//              tile's strip of vocabulary columns (Eq. 1's log pi: log-softmax at the sampled
 //              token, plus entropy and argmax). The logits never leave the SM.
 //   role DZ  : the same product recomputed, turned in registers into
 //              dz = g_t (onehot(y_t) - exp(z - lse_t)) and stored as bf16 (one vocab chunk).
@@ -34,10 +34,29 @@ constexpr int BK = 64;         // one 128-byte swizzle row of bf16
 constexpr uint32_t BOX_MN = 64 * 64 * 2;   // one 64 x 64 bf16 box (MN-major operands)
 constexpr uint32_t TMEM_COLS = 512;        // two 128 x 256 f32 accumulators
 constexpr int NUM_THREADS = 192;
-#ifndef GRPO_GROUP_M
-#define GRPO_GROUP_M 16
+// Raster groups: row tiles that consecutive work units walk before moving to the next column
+// unit, per role. Measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
+// V = 151936 (step time against the neighbouring values): forward 16 (8: +7 %, 32: +0.5 %),
+// dz recompute 32 (16: +1.5 %, 64: +15 %), dH and dW 64 (16: +7 %, 32: +2 %, 128: +0.5 %).
+#ifndef GRPO_GROUP_M_FWD
+#define GRPO_GROUP_M_FWD 16
 #endif
-constexpr int GROUP_M = GRPO_GROUP_M;      // raster: row units sharing each column sweep
+#ifndef GRPO_GROUP_M_DZ
+#define GRPO_GROUP_M_DZ 32
+#endif
+#ifndef GRPO_GROUP_M_DH
+#define GRPO_GROUP_M_DH 64
+#endif
+#ifndef GRPO_GROUP_M_DW
+#define GRPO_GROUP_M_DW 64
+#endif
+template <int ROLE>
+constexpr int group_rows() {
+  return ROLE == ROLE_FWD || ROLE == ROLE_FWD_KL ? GRPO_GROUP_M_FWD
+         : ROLE == ROLE_DZ || ROLE == ROLE_DZ_KL ? GRPO_GROUP_M_DZ
+         : ROLE == ROLE_DH                       ? GRPO_GROUP_M_DH
+                                                 : GRPO_GROUP_M_DW;
+}
 
 // Tile modes (MODE template parameter):
 //   0 single CTA : one CTA computes a 128 x 256 tile (tcgen05 cta_group::1, M = 128); two
@@ -130,7 +149,7 @@ __device__ __forceinline__ int acc_tiles_of_unit(const GemmArgs& a, int n) {
 // Work layout shared by the three roles of a CTA. In the pair modes a unit is the 2 consecutive
 // row tiles of a pair (2*mu + rank for CTA `rank`) with one column unit of NT 256-column tiles,
 // and units are strided over the resident pairs.
-template <int MODE>
+template <int ROLE, int MODE>
 struct Sched {
   int rank;        // CTA rank in the cluster (pair modes: 0 = leader, issues the MMAs); 0 in mode 0
   int group;       // row units per raster group
@@ -145,7 +164,7 @@ struct Sched {
     step = static_cast<int>(gridDim.x) / CL;
     num_mu = (dm.num_m + CL - 1) / CL;
     num_nu = (dm.num_n + NT - 1) / NT;
-    group = GROUP_M / CL > 0 ? GROUP_M / CL : 1;   // GROUP_M row tiles per raster group
+    group = group_rows<ROLE>() / CL > 0 ? group_rows<ROLE>() / CL : 1;   // in row units
     num_units = num_mu * num_nu;
   }
   // Unit u -> the row tile m this CTA stages (always a valid tile), the column unit n, and
@@ -168,10 +187,13 @@ struct Sched {
 // shared by the CTAs working on its other column tiles, or a column tile of B shared by the
 // CTAs on other row tiles) find it in L2 only if they read it within a few tens of microseconds
 // of one another: the L2 turns over that fast under these kernels' traffic. Over the thousands
-// of k-blocks of a long-K unit, CTAs otherwise drift apart by more than that. So every
-// `check` k-blocks the producer of each CTA counts itself in and waits until the CTAs of the
-// launch have, on average, reached `lag` checkpoints behind it. The slowest CTA never waits, so
-// the window cannot deadlock. It is a hint: a wait that runs past its bound switches the
+// of k-blocks of a long-K unit, and over the successive units a CTA takes in turn, CTAs
+// otherwise drift apart by more than that. So at every checkpoint the producer of each CTA
+// counts itself in and waits until the CTAs of the launch have, on average, reached `lag`
+// checkpoints behind it. Checkpoints fall every `check` k-blocks (check > 0) or at the start of
+// every -check-th work unit (check < 0: with lag 1, a barrier between the waves of units, so
+// the drift never outlasts one unit and no wait falls inside one). The slowest CTA never waits,
+// so the window cannot deadlock. It is a hint: a wait that runs past its bound switches the
 // window off for this CTA, and a CTA that leaves adds 2^40 so that no one waits for it.
 struct ProgressWindow {
   unsigned long long* arrivals;
@@ -181,10 +203,9 @@ struct ProgressWindow {
   bool on;
   __device__ __forceinline__ ProgressWindow(const GemmArgs& a)
       : arrivals(&a.hdr->win_arrivals), exited(&a.hdr->win_exited), grid(gridDim.x),
-        check(a.win_check), lag(a.win_lag), on(a.win_check > 0 && a.win_lag > 0) {}
-  __device__ __forceinline__ void at(long long kblocks_issued) {
-    if (!on || kblocks_issued == 0 || kblocks_issued % check != 0) return;
-    const long long c = kblocks_issued / check;
+        check(a.win_check), lag(a.win_lag), on(a.win_check != 0 && a.win_lag > 0) {}
+  // Checkpoint number c reached: count in, then wait for the launch's average.
+  __device__ __forceinline__ void arrive_and_wait(long long c) {
     atomicAdd(arrivals, 1ull);
     if (c < lag) return;
     const unsigned long long target = grid * static_cast<unsigned long long>(c - lag + 1);
@@ -196,6 +217,16 @@ struct ProgressWindow {
       }
       __nanosleep(64);
     }
+  }
+  // Before issuing k-block number `kblocks_issued` (counted over the whole launch).
+  __device__ __forceinline__ void at(long long kblocks_issued) {
+    if (!on || check <= 0 || kblocks_issued == 0 || kblocks_issued % check != 0) return;
+    arrive_and_wait(kblocks_issued / check);
+  }
+  // Before the first k-block of this CTA's work unit number `units_started` (0, 1, ...).
+  __device__ __forceinline__ void at_unit(long long units_started) {
+    if (!on || check >= 0 || units_started == 0 || units_started % (-check) != 0) return;
+    arrive_and_wait(units_started / (-check));
   }
   __device__ __forceinline__ void leave() {
     atomicAdd(arrivals, 1ull << 40);
@@ -210,7 +241,7 @@ struct ProgressWindow {
 template <int ROLE, int MODE>
 __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
                              const CUtensorMap* mapA2, const CUtensorMap* mapB2, const GemmArgs& a,
-                             const Dims& dm, const Sched<MODE>& sc, uint8_t* sA, uint8_t* sB,
+                             const Dims& dm, const Sched<ROLE, MODE>& sc, uint8_t* sA, uint8_t* sB,
                              uint64_t* full, uint64_t* empty, volatile int* abort_flag) {
   using C = Cfg<MODE>;
   constexpr bool PAIR = C::PAIR;
@@ -225,10 +256,12 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
   long long issued = 0;
   bool ok = true;
   ProgressWindow win(a);
+  long long units_started = 0;
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
     int m_load, n;
     bool m_ok;
     sc.decode(u, dm, m_load, n, m_ok);
+    win.at_unit(units_started++);
     const int nacc = acc_tiles_of_unit<ROLE>(a, n);
     const int hrow = m_load * BM;   // first packed row of the tile (FWD / DZ / KL A operand)
     // The boxes of k-block kbi of accumulator tile ti: fa / fb(smem offset, map, x, y) for each
@@ -347,7 +380,7 @@ struct OneBuf {
 };
 
 template <int ROLE, int MODE>
-__device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc, uint8_t* sA,
+__device__ void run_mma(const GemmArgs& a, const Dims& dm, const Sched<ROLE, MODE>& sc, uint8_t* sA,
                         uint8_t* sB, uint64_t* full, uint64_t* empty, uint64_t* accf,
                         uint64_t* acce, uint64_t* drain, uint32_t tmem_base,
                         volatile int* abort_flag) {
@@ -484,7 +517,7 @@ __device__ __forceinline__ void advance_buf(uint32_t& buf, uint32_t& bphase) {
 }
 
 template <int ROLE, int MODE>
-__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<MODE>& sc,
+__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE, MODE>& sc,
                              uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
                              volatile int* abort_flag) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -885,7 +918,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const Dims dm = role_dims<ROLE>(args, args.hdr->num_tiles);
-  const Sched<MODE> sc(dm);
+  const Sched<ROLE, MODE> sc(dm);
 
   if (warp == 0) {
     if (lane == 0)

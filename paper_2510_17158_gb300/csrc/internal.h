@@ -18,8 +18,15 @@ struct WsHeader;
 constexpr int kTileRows = 128;
 // Vocabulary tile (N of the forward and dz GEMMs) and hidden tile (N of the dH / dW GEMMs).
 constexpr int kTileN = 256;
-// Vocabulary tiles merged on chip by one forward work unit before it writes partial statistics.
-constexpr int kFwdTilesPerStrip = 8;
+// Vocabulary tiles merged on chip by one forward work unit before it writes partial statistics
+// (a strip). One tile per unit: CTAs that read the same W tile then start and finish it together
+// (longer strips let them drift apart and re-read W from HBM: 8-tile strips ran the forward
+// GEMM 6-9 % slower at the 2 x 16, T = 16384, d = 5120 workload), at the price of 16 bytes of
+// statistics per token and 256 vocabulary columns for the merge to read back.
+#ifndef GRPO_FWD_TILES_PER_STRIP
+#define GRPO_FWD_TILES_PER_STRIP 1
+#endif
+constexpr int kFwdTilesPerStrip = GRPO_FWD_TILES_PER_STRIP;
 
 // FWD_KL / DZ_KL: the forward / dz roles with a second product z_ref = W_ref h_ref (the frozen
 // reference model) in the other half of tensor memory, for Eq. 1's exact KL term.

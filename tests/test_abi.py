@@ -73,8 +73,9 @@ def test_host_validation_rejects_before_launch(lib):
 
 def test_process_wide_settings_validate_and_round_trip(lib):
     """Host-only setters (no GPU work): tile modes 0 and 1 accepted for every role at once and
-    read back, others refused (mode 2 is per-role only); the progress window refuses negative
-    values and a checkpoint with lag 0; the CTA-pair switch maps to tile modes 1 / 0."""
+    read back, others refused (mode 2 is per-role only); the progress window refuses a negative
+    lag and a checkpoint with lag 0, and takes negative checkpoint spacings (in work units); the
+    CTA-pair switch maps to tile modes 1 / 0."""
     try:
         for mode in (0, 1):
             assert lib.grpo_set_tile_mode(mode) == 0
@@ -87,10 +88,12 @@ def test_process_wide_settings_validate_and_round_trip(lib):
         assert lib.grpo_set_cta_pair(1) == 0 and lib.grpo_get_tile_mode() == 1
     finally:
         lib.grpo_set_tile_mode(-1)
-    assert lib.grpo_set_gemm_window(-1, 2) == -1
     assert lib.grpo_set_gemm_window(16, -1) == -1
     assert lib.grpo_set_gemm_window(16, 0) == -1
+    assert lib.grpo_set_gemm_window(-1, 0) == -1
     assert lib.grpo_set_gemm_window(16, 4) == 0
+    assert lib.grpo_set_gemm_window(-1, 1) == 0      # checkpoints at every unit start
+    assert lib.grpo_set_gemm_window(-2, 2) == 0
     assert lib.grpo_set_gemm_window(0, 0) == 0
 
 

@@ -207,15 +207,16 @@ def test_chunked_backward_full_vocabulary_partial_last_chunk():
 
 def test_progress_window_changes_nothing_and_resets_its_counters():
     """The GEMM progress window only delays TMA issue: outputs with it off (the default), at 16
-    k-blocks with lag 4 and at a tight setting (1 k-block, lag 1, so that the producers wait at
-    every k-block) are bitwise equal, and the last CTA of every launch resets the window's
+    k-blocks with lag 4, at a tight setting (1 k-block, lag 1, so that the producers wait at
+    every k-block) and with checkpoints at every work unit's start (-1, lag 1: a barrier between
+    waves of units) are bitwise equal, and the last CTA of every launch resets the window's
     counters in the workspace header (arrivals at byte 24, CTAs left at byte 32) to 0."""
     from paper_2510_17158_gb300 import grpo as G
     b = _batch("d4096_v152k")
     old, ref = oracle_inputs(b)
     outs = []
     try:
-        for check, lag in ((0, 0), (16, 4), (1, 1)):
+        for check, lag in ((0, 0), (16, 4), (1, 1), (-1, 1)):
             G.grpo_set_gemm_window(check, lag)
             outs.append(run_gpu(b, old, ref, 0.2, 0.2, 0.04))
             dev = torch.device("cuda")

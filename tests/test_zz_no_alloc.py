@@ -64,11 +64,11 @@ def test_static_scratch_rejects_batches_larger_than_the_array():
 def _static_bytes(S, T, d, V):
     """Scratch the bf16 path of grpo_score_fwd_static lays out (256-byte aligned regions):
     header, sequence bases, packed-row map, position map, target logits, per-strip statistics
-    (16 bytes per packed row and 2048-column vocabulary strip) and the packed hidden states."""
+    (16 bytes per packed row and 256-column vocabulary strip) and the packed hidden states."""
     up = lambda x: (x + 255) // 256 * 256            # noqa: E731
     P = S * T
     R = (P + 127) // 128 * 128
-    strips = ((V + 255) // 256 + 7) // 8
+    strips = (V + 255) // 256
     return (256 + up(4 * (S + 1)) + up(4 * R) + up(4 * P) + up(4 * P) + up(16 * strips * R) +
             up(2 * R * d))
 
@@ -98,25 +98,31 @@ def test_static_scratch_f32_forward_matches_workspace_forward():
 
 
 def test_static_scratch_batch_just_below_the_array_size():
-    """One completion of T = 15360 tokens at d = 2048, V = 32000 needs 67,031,552 bytes of the
-    67,108,864: it runs and matches the workspace path. T = 15361 rounds up to one more 128-row
-    tile (67,589,632 bytes) and is refused before anything is enqueued."""
+    """At d = 2048, V = 32000 one completion of T = T_max tokens (the largest multiple of 128
+    whose scratch fits the 64 MiB array) runs and matches the workspace path; T_max + 1 rounds up
+    to one more 128-row tile and is refused before anything is enqueued."""
     d, V = 2048, 32000
-    assert _static_bytes(1, 15360, d, V) <= G.STATIC_SCRATCH_BYTES < _static_bytes(1, 15361, d, V)
-    assert G.STATIC_SCRATCH_BYTES - _static_bytes(1, 15360, d, V) < 128 * 1024
-    w = WORKLOADS["g8_t1k_d2048_v32k"].scaled(seed=14, prompts=1, group_sizes=(1,), T=15360,
-                                             len_lo=15000, len_hi=15360)
+    t_max = 128
+    while _static_bytes(1, t_max + 128, d, V) <= G.STATIC_SCRATCH_BYTES:
+        t_max += 128
+    assert _static_bytes(1, t_max, d, V) <= G.STATIC_SCRATCH_BYTES < _static_bytes(1, t_max + 1, d, V)
+    assert G.STATIC_SCRATCH_BYTES - _static_bytes(1, t_max, d, V) < 128 * 6200
+    w = WORKLOADS["g8_t1k_d2048_v32k"].scaled(seed=14, prompts=1, group_sizes=(1,), T=t_max,
+                                             len_lo=t_max - 300, len_hi=t_max)
     b = make_batch_torch(w, "cuda")
     H, W, tok, mask = b.H, b.W, b.tokens, b.mask
     got = G.grpo_score_fwd_static(H, W, tok, mask)
     torch.cuda.synchronize()
     assert int(got["status"].item()) == 0
     _same_as_workspace_forward(H, W, tok, mask, got)
-    lib = G._lib()
-    fake = ctypes.c_void_p(1 << 20)       # never dereferenced: the size check fails first
-    st = lib.grpo_score_fwd_static(fake, fake, G.GRPO_BF16, fake, fake, 1, 15361, d, V, fake, fake,
-                                   fake, fake, fake, ctypes.c_void_p(0), ctypes.c_void_p(0))
-    assert st == -4, G.grpo_status_string(st)
+    # one token more: real buffers of the right size, so that nothing could be read out of
+    # bounds even if the size check let the call through
+    H2 = torch.zeros((1, t_max + 1, d), dtype=torch.bfloat16, device="cuda")
+    tok2 = torch.zeros((1, t_max + 1), dtype=torch.int32, device="cuda")
+    mask2 = torch.ones((1, t_max + 1), dtype=torch.uint8, device="cuda")
+    with pytest.raises(G.GrpoError) as err:
+        G.grpo_score_fwd_static(H2, W, tok2, mask2)
+    assert err.value.status == -4, err.value
 
 
 def test_static_scratch_reports_a_bad_token_and_the_next_call_clears_it():
