@@ -314,8 +314,10 @@ def run_gpu(args):
             raise SystemExit("--role-tile-modes wants four comma-separated modes (fwd,dz,dH,dW)")
         for role, m in enumerate(role_modes):
             G.grpo_set_role_tile_mode(role, m)
-    win = [int(x) for x in args.gemm_window.split(",")]
-    G.grpo_set_gemm_window(win[0], win[1])
+    win = None
+    if args.gemm_window:
+        win = [int(x) for x in args.gemm_window.split(",")]
+        G.grpo_set_gemm_window(win[0], win[1])
     w = apply_scale(WORKLOADS[args.config], args.scale)
     w = w.scaled(seed=w.seed + 1000 * rank)        # each rank scores its own groups
     if args.beta is not None:
@@ -433,13 +435,14 @@ def run_gpu(args):
         table = {"graph_replay": (args.steps, ms)}
     dom = max(table, key=lambda k: table[k][1])
     n_dom, t_dom = table[dom]
-    chunk = args.vocab_chunk or V
     kl2 = 2.0 if args.path == "grpo-exact-kl" else 1.0
-    flops_per_launch = {
-        "fwd_gemm_tc": 2.0 * kl2 * N_v * d * V, "bwd_dz_gemm_tc": 2.0 * kl2 * N_v * d * min(V, chunk),
-        "bwd_dh_gemm_tc": 2.0 * N_v * d * min(V, chunk), "bwd_dw_gemm_tc": 2.0 * N_v * d * min(V, chunk)}
-    if dom in flops_per_launch:
-        achieved = flops_per_launch[dom] / ((t_dom / n_dom) / 1e3) / 1e12
+    # algorithmic flop of each GEMM per step, summed over its launches (one per vocabulary chunk
+    # for dz, dH and dW; the last chunk may be narrower); rates = timed-region flop / kernel time
+    flops_per_step = {
+        "fwd_gemm_tc": 2.0 * kl2 * N_v * d * V, "bwd_dz_gemm_tc": 2.0 * kl2 * N_v * d * V,
+        "bwd_dh_gemm_tc": 2.0 * N_v * d * V, "bwd_dw_gemm_tc": 2.0 * N_v * d * V}
+    if dom in flops_per_step:
+        achieved = flops_per_step[dom] * args.steps / (t_dom / 1e3) / 1e12
         roof = {"kernel": dom, "bound": "tensor", "achieved": round(achieved, 1),
                 "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
                 "frac": round(achieved / pk["bf16_sustained"], 4),
@@ -454,7 +457,7 @@ def run_gpu(args):
     for k in GEMM_KERNELS:
         if k in table:
             n, t = table[k]
-            gemm_tf[k] = round(flops_per_launch[k] / ((t / n) / 1e3) / 1e12, 1)
+            gemm_tf[k] = round(flops_per_step[k] * args.steps / (t / 1e3) / 1e12, 1)
 
     out = {
         "metric": "scored tokens/sec (fwd+bwd)" + {"sft": " [SFT distillation step]",
@@ -467,7 +470,8 @@ def run_gpu(args):
                    "d": d, "V": V, "eps": w.eps, "beta": w.beta, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
                    "tiles": tiles_desc(G),
-                   "gemm_window": ("off" if win[0] == 0 else
+                   "gemm_window": ("library default (dH, dW: checkpoint at every work unit, "
+                                   "lag 1)" if win is None else "off" if win[0] == 0 else
                                    f"{win[0]} k-blocks, lag {win[1]} checkpoints" if win[0] > 0
                                    else f"every {-win[0]} work unit(s), lag {win[1]}"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
@@ -526,10 +530,11 @@ def main():
     ap.add_argument("--role-tile-modes", default="",
                     help="per-GEMM tile modes fwd,dz,dH,dW, applied after --tile-mode "
                          "(-1 = that GEMM's default; 2 = " + TILE_MODES[2] + ", dH and dW only)")
-    ap.add_argument("--gemm-window", default="0,0",
-                    help="GEMM progress window CHECK,LAG: producers stay within LAG checkpoints of "
-                         "the launch's average; checkpoints every CHECK k-blocks, or at every "
-                         "-CHECK-th work unit for CHECK < 0 (write --gemm-window=-1,1); '0,0' = off")
+    ap.add_argument("--gemm-window", default="",
+                    help="progress window of the dH and dW GEMMs CHECK,LAG: producers stay within "
+                         "LAG checkpoints of the launch's average; checkpoints every CHECK "
+                         "k-blocks, or at every -CHECK-th work unit for CHECK < 0 (write "
+                         "--gemm-window=-1,1); '0,0' = off; default: the library's (-1,1)")
     ap.add_argument("--graph", action="store_true",
                     help="capture one step in a CUDA graph and time its replays (per-kernel "
                          "timing and launch counts then come from the capture, not the replays)")

@@ -295,15 +295,16 @@ int grpo_set_cta_pair(int32_t on);
 int grpo_set_role_tile_mode(int32_t role, int32_t mode);
 int grpo_get_role_tile_mode(int32_t role);
 
-/* Progress window of the tensor-core GEMMs, process-wide, for launches made afterwards. At every
- * checkpoint the TMA producer of each CTA waits (at most 0.5 ms) until the CTAs of the launch are
- * on average within `lag` checkpoints of it, so that CTAs reading the same operand tiles read
- * them close enough in time to hit L2 (long-K GEMMs otherwise drift apart and re-read their
- * operands from HBM). Checkpoints fall every `check_kblocks` k-blocks of 64 (check_kblocks > 0)
- * or, for check_kblocks < 0, at the start of every (-check_kblocks)-th work unit (an output
- * tile or strip): with lag 1 a barrier between the waves of units. Results do not depend on it.
- * check_kblocks == 0 turns it off (the default). Returns GRPO_ERR_INVALID_ARG for a negative lag
- * or for check_kblocks != 0 with lag == 0. */
+/* Progress window of the long-K tensor-core GEMMs (dH and dW; the forward and dz GEMMs never
+ * wait), process-wide, for launches made afterwards. At every checkpoint the TMA producer of each
+ * CTA waits (at most 0.5 ms) until the CTAs of the launch are on average within `lag`
+ * checkpoints of it, so that CTAs reading the same operand tiles read them close enough in time
+ * to hit L2 (CTAs that share a tile otherwise drift apart over successive long-K units and
+ * re-read their operands from HBM). Checkpoints fall every `check_kblocks` k-blocks of 64
+ * (check_kblocks > 0) or, for check_kblocks < 0, at the start of every (-check_kblocks)-th work
+ * unit (an output tile): with lag 1 a barrier between the waves of units. Default (-1, 1).
+ * Results do not depend on it. check_kblocks == 0 turns it off. Returns GRPO_ERR_INVALID_ARG
+ * for a negative lag or for check_kblocks != 0 with lag == 0. */
 int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag);
 
 #ifdef __cplusplus

@@ -36,10 +36,11 @@ constexpr uint32_t TMEM_COLS = 512;        // two 128 x 256 f32 accumulators
 constexpr int NUM_THREADS = 192;
 // Raster groups: row tiles that consecutive work units walk before moving to the next column
 // unit, per role. Measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
-// V = 151936 (step time against the neighbouring values): forward 16 (8: +7 %, 32: +0.5 %),
-// dz recompute 32 (16: +1.5 %, 64: +15 %), dH and dW 64 (16: +7 %, 32: +2 %, 128: +0.5 %).
+// V = 151936 (the GEMM's time against the neighbouring values): forward 32 (16: +0-2 %,
+// 8: +7 %), dz recompute 32 (16: +1.5 %, 64: +15 %), dH and dW 64 (16: +7 %, 32: +2 %, 128:
+// +0.5 %, measured without the progress window).
 #ifndef GRPO_GROUP_M_FWD
-#define GRPO_GROUP_M_FWD 16
+#define GRPO_GROUP_M_FWD 32
 #endif
 #ifndef GRPO_GROUP_M_DZ
 #define GRPO_GROUP_M_DZ 32
@@ -201,9 +202,11 @@ struct ProgressWindow {
   unsigned long long grid;
   int check, lag;
   bool on;
-  __device__ __forceinline__ ProgressWindow(const GemmArgs& a)
+  // `long_k`: the window applies to the long-K roles (dH, dW) only; the forward and dz GEMMs,
+  // whose units are one short tile, never wait (a barrier there costs 3-4 % and saves nothing).
+  __device__ __forceinline__ ProgressWindow(const GemmArgs& a, bool long_k)
       : arrivals(&a.hdr->win_arrivals), exited(&a.hdr->win_exited), grid(gridDim.x),
-        check(a.win_check), lag(a.win_lag), on(a.win_check != 0 && a.win_lag > 0) {}
+        check(a.win_check), lag(a.win_lag), on(long_k && a.win_check != 0 && a.win_lag > 0) {}
   // Checkpoint number c reached: count in, then wait for the launch's average.
   __device__ __forceinline__ void arrive_and_wait(long long c) {
     atomicAdd(arrivals, 1ull);
@@ -255,7 +258,7 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
   uint32_t stage = 0, phase = 0;
   long long issued = 0;
   bool ok = true;
-  ProgressWindow win(a);
+  ProgressWindow win(a, ROLE == ROLE_DH || ROLE == ROLE_DW);
   long long units_started = 0;
   for (int u = sc.first; u < sc.num_units && ok; u += sc.step) {
     int m_load, n;

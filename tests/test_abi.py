@@ -95,6 +95,7 @@ def test_process_wide_settings_validate_and_round_trip(lib):
     assert lib.grpo_set_gemm_window(-1, 1) == 0      # checkpoints at every unit start
     assert lib.grpo_set_gemm_window(-2, 2) == 0
     assert lib.grpo_set_gemm_window(0, 0) == 0
+    assert lib.grpo_set_gemm_window(-1, 1) == 0      # back to the library's default
 
 
 def test_role_tile_modes_defaults_overrides_and_refusals(lib):

@@ -206,11 +206,11 @@ def test_chunked_backward_full_vocabulary_partial_last_chunk():
 
 
 def test_progress_window_changes_nothing_and_resets_its_counters():
-    """The GEMM progress window only delays TMA issue: outputs with it off (the default), at 16
-    k-blocks with lag 4, at a tight setting (1 k-block, lag 1, so that the producers wait at
+    """The progress window of the dH and dW GEMMs only delays TMA issue: outputs with it off, at
+    16 k-blocks with lag 4, at a tight setting (1 k-block, lag 1, so that the producers wait at
     every k-block) and with checkpoints at every work unit's start (-1, lag 1: a barrier between
-    waves of units) are bitwise equal, and the last CTA of every launch resets the window's
-    counters in the workspace header (arrivals at byte 24, CTAs left at byte 32) to 0."""
+    waves of units, the default) are bitwise equal, and the last CTA of every launch resets the
+    window's counters in the workspace header (arrivals at byte 24, CTAs left at byte 32) to 0."""
     from paper_2510_17158_gb300 import grpo as G
     b = _batch("d4096_v152k")
     old, ref = oracle_inputs(b)
@@ -223,13 +223,17 @@ def test_progress_window_changes_nothing_and_resets_its_counters():
             H, W = b.H.to(dev), b.W.to(dev)
             S, T, d = H.shape
             ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype)
-            G.grpo_score_fwd(H, W, b.tokens.to(dev), b.mask.to(dev), ws)
+            tok, mask = b.tokens.to(dev), b.mask.to(dev)
+            f = G.grpo_score_fwd(H, W, tok, mask, ws)
+            adv = G.group_advantages(b.rewards.to(dev), b.group_offsets.to(dev), ws)
+            G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], torch.from_numpy(old).to(dev),
+                            torch.from_numpy(ref).to(dev), adv, f["valid_count"], ws)
             torch.cuda.synchronize()
             hdr = ws.buf[:64].cpu().numpy()
             assert int(hdr[24:32].view(np.uint64)[0]) == 0
             assert int(hdr[32:36].view(np.uint32)[0]) == 0
     finally:
-        G.grpo_set_gemm_window(0, 0)
+        G.grpo_set_gemm_window(-1, 1)
     for g in outs[1:]:
         for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
             assert torch.equal(g[k], outs[0][k]), k
