@@ -488,7 +488,7 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   // exact-KL roles: single-CTA tiles
   const int tm = mode == 2 ? 0 : gemm_role_tile_mode(ROLE_DZ);
   const int tm_dh = gemm_role_tile_mode(ROLE_DH), tm_dw = gemm_role_tile_mode(ROLE_DW);
-  CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn, mapHrk, mapWrk;
+  CUtensorMap mapHk, mapWk, mapDzK, mapWmn, mapDzMn, mapHmn, mapHrk, mapWrk, mapDzSt;
   if (mode == 2 && (!make_map(&mapHrk, v.hrp, d, L.rows_cap, d, kTileRows) ||
                     !make_map(&mapWrk, W_ref, d, V, d, kTileN)))
     return GRPO_ERR_CUDA;
@@ -496,7 +496,9 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
       !make_map(&mapWk, W, d, V, d, gemm_b_box_rows(tm)) ||
       !make_map(&mapDzK, dz, vc, L.rows_cap, vc, kTileRows) ||
       !make_map(&mapWmn, W, d, V, d, 64) || !make_map(&mapDzMn, dz, vc, L.rows_cap, vc, 64) ||
-      !make_map(&mapHmn, v.hp, d, L.rows_cap, d, 64))
+      !make_map(&mapHmn, v.hp, d, L.rows_cap, d, 64) ||
+      // single-CTA dz tiles store 32-row x 64-column boxes of dz through this map
+      !make_map(&mapDzSt, dz, vc, L.rows_cap, vc, 32))
     return GRPO_ERR_CUDA;
 
   GemmArgs a = base_args(L, v, S, T, d, V, tokens, mask);
@@ -522,7 +524,8 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
       if (mode == 2)
         return launch_gemm(ROLE_DZ_KL, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, 0), 0, st,
                            &mapHrk, &mapWrk);
-      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, tm), tm, st);
+      return launch_gemm(ROLE_DZ, mapHk, mapWk, a, gemm_grid(L.max_tiles, vt, tm), tm, st,
+                         &mapDzSt);
     }));
     GRPO_TRY(counted(GRPO_K_BWD_DH_GEMM, st, [&] {
       return launch_gemm(ROLE_DH, mapDzK, mapWmn, a, gemm_grid(L.max_tiles, dtiles, tm_dh),

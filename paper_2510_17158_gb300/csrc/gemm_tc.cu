@@ -87,8 +87,22 @@ struct Cfg {
   static constexpr uint32_t STAGE_TX = A_STAGE + B_STAGE;   // bytes landing per CTA
   static constexpr size_t SMEM = size_t(STAGES) * STAGE_TX + 1024 + 256;
 };
+// Shared-memory staging of the dz tile for its TMA stores (single-CTA dz only): per epilogue warp
+// two buffers of 32 rows x 64 bf16 columns (4 KB, rows of 128 bytes in the 128-byte swizzle), so
+// that a warp fills one while the TMA engine reads the other.
+template <int ROLE, int MODE>
+struct OutStage {
+  static constexpr bool on = MODE == 0 && ROLE == ROLE_DZ;
+  static constexpr uint32_t BUF = 32 * 64 * 2;
+  static constexpr uint32_t BYTES = on ? 4 * 2 * BUF : 0;
+};
+template <int ROLE, int MODE>
+constexpr size_t smem_bytes() {
+  return Cfg<MODE>::SMEM + OutStage<ROLE, MODE>::BYTES;
+}
 constexpr size_t smax(size_t a, size_t b) { return a > b ? a : b; }
-constexpr size_t SMEM_BYTES = smax(Cfg<0>::SMEM, smax(Cfg<1>::SMEM, Cfg<2>::SMEM));
+constexpr size_t SMEM_BYTES =
+    smax(smem_bytes<ROLE_DZ, 0>(), smax(Cfg<0>::SMEM, smax(Cfg<1>::SMEM, Cfg<2>::SMEM)));
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory per CTA");
 
 struct Dims {
@@ -520,9 +534,10 @@ __device__ __forceinline__ void advance_buf(uint32_t& buf, uint32_t& bphase) {
 }
 
 template <int ROLE, int MODE>
-__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE, MODE>& sc,
-                             uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
-                             volatile int* abort_flag) {
+__device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sched<ROLE, MODE>& sc,
+                                   uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
+                                   volatile int* abort_flag, uint8_t* s_out,
+                                   const CUtensorMap* map_out) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;               // TMEM lane quadrant this warp may access
   const int r = q * 32 + lane;          // accumulator row of this thread
@@ -530,6 +545,7 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE
   const int32_t where = WHERE_GEMM_BASE + ROLE * 16 + 4;
   constexpr int NT = Cfg<MODE>::NT;   // 256-column halves of the accumulator tile
   uint32_t buf = 0, bphase = 0;
+  uint32_t ob = 0;                    // dz staging buffer this warp fills next (TMA-store path)
   for (int u = sc.first; u < sc.num_units; u += sc.step) {
     int m_load, n;
     bool m_ok;   // this CTA stores the tile (false: a pair's second CTA past the last tile)
@@ -753,15 +769,11 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE
       const int y = act ? a.tokens[pos] - a.v_offset : -1;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
-      __nv_bfloat16* dst_row =
-          a.dz + (static_cast<size_t>(m_load) * BM + r) * static_cast<size_t>(a.dz_pitch);
-      for (int c = 0; c < BN / 32; ++c) {
-        const int vloc = n * BN + c * 32;
-        const int v0 = a.vc0 + vloc;
+      // dz of 32 consecutive columns of this row, bf16 pairs, from accumulator columns c*32..
+      auto dz_chunk = [&](int c, uint32_t (&pk)[16]) {
+        const int v0 = a.vc0 + n * BN + c * 32;
         float x[32];
         tmem_load_32cols(t_row + buf * BN + c * 32, x);
-        if (!m_ok) continue;
-        uint32_t pk[16];
         if (act) {
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -776,10 +788,46 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE
 #pragma unroll
           for (int j = 0; j < 16; ++j) pk[j] = 0u;
         }
-        uint4* dst = reinterpret_cast<uint4*>(dst_row + vloc);
+      };
+      if constexpr (OutStage<ROLE, MODE>::on) {
+        // 64 columns at a time: the warp's 32 rows go to a 4 KB staging buffer (row = lane,
+        // 16-byte chunk j stored at chunk j ^ (row % 8): the 128-byte swizzle of the store's
+        // tensor map), then one TMA store writes them as full 128-byte row segments.
+        for (int c2 = 0; c2 < BN / 64; ++c2) {
+          uint32_t lo[16], hi[16];
+          dz_chunk(2 * c2, lo);
+          dz_chunk(2 * c2 + 1, hi);
+          uint8_t* stage = s_out + (q * 2 + ob) * OutStage<ROLE, MODE>::BUF;
+          if (lane == 0) bulk_wait_group_read<1>();   // this buffer's previous store has read it
+          __syncwarp();
+          uint8_t* row = stage + lane * 128;
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+          for (int j = 0; j < 8; ++j) {
+            const uint32_t* p = j < 4 ? &lo[4 * j] : &hi[4 * (j - 4)];
+            *reinterpret_cast<uint4*>(row + ((j ^ (lane & 7)) << 4)) =
+                make_uint4(p[0], p[1], p[2], p[3]);
+          }
+          fence_proxy_async_smem();   // make the writes visible to the TMA engine
+          __syncwarp();
+          if (lane == 0 && m_ok) {
+            tma_store_2d(map_out, smem_u32(stage), n * BN + c2 * 64, m_load * BM + q * 32);
+            bulk_commit_group();
+          }
+          ob ^= 1u;
+        }
+      } else {
+        __nv_bfloat16* dst_row =
+            a.dz + (static_cast<size_t>(m_load) * BM + r) * static_cast<size_t>(a.dz_pitch);
+        for (int c = 0; c < BN / 32; ++c) {
+          const int vloc = n * BN + c * 32;
+          uint32_t pk[16];
+          dz_chunk(c, pk);
+          if (!m_ok) continue;
+          uint4* dst = reinterpret_cast<uint4*>(dst_row + vloc);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+        }
       }
       epi_release<MODE>(&acce[buf], lane, sc.rank);
       buf ^= 1u;
@@ -857,6 +905,17 @@ __device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE
   }
 }
 
+template <int ROLE, int MODE>
+__device__ void run_epilogue(const GemmArgs& a, const Dims& dm, const Sched<ROLE, MODE>& sc,
+                             uint64_t* accf, uint64_t* acce, uint32_t tmem_base,
+                             volatile int* abort_flag, uint8_t* s_out,
+                             const CUtensorMap* map_out) {
+  run_epilogue_tiles<ROLE, MODE>(a, dm, sc, accf, acce, tmem_base, abort_flag, s_out, map_out);
+  // TMA-store path: the issuing lane's stores must have written global memory (and finished
+  // reading the staging buffers) before the CTA leaves
+  if (OutStage<ROLE, MODE>::on && (threadIdx.x & 31) == 0) bulk_wait_group_all();
+}
+
 // ------------------------------------------------------------------------------------------
 // kernel body (every tile mode) and one kernel per mode
 // ------------------------------------------------------------------------------------------
@@ -871,7 +930,8 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_STAGE;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_STAGE);
+  uint8_t* sOut = sB + C::STAGES * C::B_STAGE;   // dz staging (OutStage), 1024-byte aligned
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sOut + OutStage<ROLE, MODE>::BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + C::STAGES;
   uint64_t* accf = bars + 2 * C::STAGES;
@@ -902,6 +962,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
       tma_prefetch_desc(mapA2);
       tma_prefetch_desc(mapB2);
     }
+    if (OutStage<ROLE, MODE>::on) tma_prefetch_desc(mapA2);   // the dz store map
   }
   if (warp == 1) {
     if (PAIR) {
@@ -932,7 +993,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
       run_mma<ROLE, MODE>(args, dm, sc, sA, sB, full, empty, accf, acce, drain, tmem_base,
                           abort_flag);
   } else {
-    run_epilogue<ROLE, MODE>(args, dm, sc, accf, acce, tmem_base, abort_flag);
+    run_epilogue<ROLE, MODE>(args, dm, sc, accf, acce, tmem_base, abort_flag, sOut, mapA2);
   }
   __syncwarp();
   tc_fence_before();
@@ -983,14 +1044,17 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
                         const CUtensorMap& mapB2) {
   if constexpr (!Dual<ROLE>::value) {       // exact-KL roles: single-CTA tiles only
     if (mode == 1)
-      return launch_with_smem(tc_gemm_pair<ROLE, 1>, Cfg<1>::SMEM, grid, st, mapA, mapB, args);
+      return launch_with_smem(tc_gemm_pair<ROLE, 1>, smem_bytes<ROLE, 1>(), grid, st, mapA, mapB,
+                              args);
     if constexpr (ROLE == ROLE_DH || ROLE == ROLE_DW) {   // wide pair: the long-K roles only
       if (mode == 2)
-        return launch_with_smem(tc_gemm_pair<ROLE, 2>, Cfg<2>::SMEM, grid, st, mapA, mapB, args);
+        return launch_with_smem(tc_gemm_pair<ROLE, 2>, smem_bytes<ROLE, 2>(), grid, st, mapA,
+                                mapB, args);
     }
   }
   if (mode != 0) return cudaErrorInvalidValue;
-  return launch_with_smem(tc_gemm<ROLE>, Cfg<0>::SMEM, grid, st, mapA, mapB, mapA2, mapB2, args);
+  return launch_with_smem(tc_gemm<ROLE>, smem_bytes<ROLE, 0>(), grid, st, mapA, mapB, mapA2,
+                          mapB2, args);
 }
 
 }  // namespace
@@ -1060,7 +1124,9 @@ cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& ma
   const CUtensorMap& b2 = mapB2 ? *mapB2 : mapB;
   switch (role) {
     case ROLE_FWD: return launch_role<ROLE_FWD>(mapA, mapB, args, grid, mode, st, a2, b2);
-    case ROLE_DZ: return launch_role<ROLE_DZ>(mapA, mapB, args, grid, mode, st, a2, b2);
+    case ROLE_DZ:   // single-CTA tiles store dz through mapA2 (the dz scratch, 64 x 32 boxes)
+      if (mode == 0 && !mapA2) return cudaErrorInvalidValue;
+      return launch_role<ROLE_DZ>(mapA, mapB, args, grid, mode, st, a2, b2);
     case ROLE_DH: return launch_role<ROLE_DH>(mapA, mapB, args, grid, mode, st, a2, b2);
     case ROLE_DW: return launch_role<ROLE_DW>(mapA, mapB, args, grid, mode, st, a2, b2);
     case ROLE_FWD_KL:
