@@ -523,13 +523,13 @@ def main():
     ap.add_argument("--path", default="grpo", choices=["grpo", "sft", "grpo-exact-kl"],
                     help="grpo: the GRPO update (default); sft: the distillation loss step; "
                          "grpo-exact-kl: GRPO with the full-vocabulary KL to a reference model")
-    ap.add_argument("--tile-mode", type=int, default=-1, choices=[-1, 0, 1],
+    ap.add_argument("--tile-mode", type=int, default=-1, choices=[-1, 0, 1, 2],
                     help="tensor-core tiles of every GEMM: -1 = the library's per-GEMM default "
                          "(fwd 0, dz 0, dH 2, dW 2); "
-                         + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items() if k < 2))
+                         + "; ".join(f"{k} = {v}" for k, v in TILE_MODES.items()))
     ap.add_argument("--role-tile-modes", default="",
                     help="per-GEMM tile modes fwd,dz,dH,dW, applied after --tile-mode "
-                         "(-1 = that GEMM's default; 2 = " + TILE_MODES[2] + ", dH and dW only)")
+                         "(-1 = that GEMM's default)")
     ap.add_argument("--gemm-window", default="",
                     help="progress window of the dH and dW GEMMs CHECK,LAG: producers stay within "
                          "LAG checkpoints of the launch's average; checkpoints every CHECK "

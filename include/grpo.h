@@ -260,23 +260,24 @@ int grpo_debug_inject_stall(int32_t on);
 /* Tensor-core tile mode of the four LM-head GEMM roles, process-wide, for launches made
  * afterwards (the exact-KL GEMMs always use single-CTA tiles). Every mode sums each output
  * element over K in the same k-block order; modes 1 and 2 issue the same M = 256 MMAs and give
- * bitwise identical dH and dW, and agree with mode 0 (M = 128 MMAs) within rounding. Every TMA
+ * bitwise identical results in every role, and agree with mode 0 (M = 128 MMAs) within rounding. Every TMA
  * copy lands in the issuing CTA's own shared memory (no multicast).
  *   GRPO_TILE_SINGLE        (0): one CTA per 128 x 256 tile (tcgen05 cta_group::1), two TMEM
  *                           accumulators (a tile's epilogue overlaps the next tile's MMAs).
  *   GRPO_TILE_CTA_PAIR      (1): clusters of two CTAs on one TPC compute 256 x 256 tiles with
  *                           cta_group::2, each CTA staging its 128 rows of A and half of B.
- *   GRPO_TILE_CTA_PAIR_WIDE (2): dH and dW only. The CTA pair computes 256 x 512 tiles: two
- *                           N = 256 MMAs per k-step into one 512-column accumulator, each CTA
- *                           staging 128 rows of A and 256 rows of B per k-block, i.e. half of
- *                           mode 0's operand bytes per flop.
+ *   GRPO_TILE_CTA_PAIR_WIDE (2): the CTA pair computes 256 x 512 tiles: two N = 256 MMAs per
+ *                           k-step into one 512-column accumulator, each CTA staging 128 rows
+ *                           of A and 256 rows of B per k-block, i.e. half of mode 0's operand
+ *                           bytes per flop; eight epilogue warps each read one half. Made for
+ *                           the long-K roles dH and dW; a forward or dz work unit is then two
+ *                           vocabulary tiles.
  *   GRPO_TILE_DEFAULT      (-1): the library's per-role choice, in force at load: the forward
  *                           product and the dz recompute in mode 0, dH and dW in mode 2.
  * Roles: GRPO_ROLE_FWD (forward scoring product), GRPO_ROLE_DZ (its recompute into dz),
  * GRPO_ROLE_DH, GRPO_ROLE_DW.
- * grpo_set_tile_mode(m) puts every role in mode m (m = -1: each role's default; m = 0 or 1);
- * grpo_set_role_tile_mode(r, m) sets one role (m = -1: that role's default; m = 2 for GRPO_ROLE_DH
- * and GRPO_ROLE_DW only).
+ * grpo_set_tile_mode(m) puts every role in mode m (m = -1: each role's default);
+ * grpo_set_role_tile_mode(r, m) sets one role (m = -1: that role's default).
  * grpo_get_tile_mode returns the mode all four roles share, or -1 when they differ (as they do
  * by default); grpo_get_role_tile_mode returns the mode role r runs in.
  * grpo_set_cta_pair(on) is grpo_set_tile_mode(on ? 1 : 0).

@@ -768,8 +768,7 @@ int grpo_debug_inject_stall(int32_t on) {
 }
 
 int grpo_set_tile_mode(int32_t mode) {
-  if (mode != GRPO_TILE_DEFAULT && mode != GRPO_TILE_SINGLE && mode != GRPO_TILE_CTA_PAIR)
-    return GRPO_ERR_INVALID_ARG;
+  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_CTA_PAIR_WIDE) return GRPO_ERR_INVALID_ARG;
   for (int r = GRPO_ROLE_FWD; r <= GRPO_ROLE_DW; ++r)
     g_role_mode[r].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[r] : mode);
   return GRPO_OK;
@@ -788,10 +787,7 @@ int grpo_get_tile_mode(void) {
 
 int grpo_set_role_tile_mode(int32_t role, int32_t mode) {
   if (role < GRPO_ROLE_FWD || role > GRPO_ROLE_DW) return GRPO_ERR_INVALID_ARG;
-  const bool long_k = role == GRPO_ROLE_DH || role == GRPO_ROLE_DW;
-  if (mode != GRPO_TILE_DEFAULT && mode != GRPO_TILE_SINGLE && mode != GRPO_TILE_CTA_PAIR &&
-      !(long_k && mode == GRPO_TILE_CTA_PAIR_WIDE))
-    return GRPO_ERR_INVALID_ARG;
+  if (mode < GRPO_TILE_DEFAULT || mode > GRPO_TILE_CTA_PAIR_WIDE) return GRPO_ERR_INVALID_ARG;
   g_role_mode[role].store(mode == GRPO_TILE_DEFAULT ? kRoleDefault[role] : mode);
   return GRPO_OK;
 }

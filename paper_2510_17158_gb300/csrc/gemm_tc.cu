@@ -33,7 +33,7 @@ constexpr int BN = kTileN;     // 256
 constexpr int BK = 64;         // one 128-byte swizzle row of bf16
 constexpr uint32_t BOX_MN = 64 * 64 * 2;   // one 64 x 64 bf16 box (MN-major operands)
 constexpr uint32_t TMEM_COLS = 512;        // two 128 x 256 f32 accumulators
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 192;          // 6 warps (modes 0, 1); mode 2: Cfg<2>::THREADS
 // Raster groups: row tiles that consecutive work units walk before moving to the next column
 // unit, per role. Measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
 // V = 151936 (the GEMM's time against the neighbouring values): forward 32 (16: +0-2 %,
@@ -69,15 +69,21 @@ constexpr int group_rows() {
 //   2 wide pair  : the CTA pair computes a 256 x 512 tile: per k-step two N = 256 MMAs write the
 //                  two 256-column halves of one 512-column accumulator. Each CTA stages 128 rows
 //                  of A and 2 x 128 rows of B per k-block (48 KB), i.e. half of mode 0's operand
-//                  bytes per flop. The epilogue does not overlap the next tile's MMAs, which is
-//                  negligible for the long-K roles DH and DW (the only roles this mode serves:
-//                  thousands of k-blocks per tile against one epilogue).
+//                  bytes per flop; eight epilogue warps each read one half. The epilogue does not
+//                  overlap the next tile's MMAs, which is negligible for the long-K roles DH and
+//                  DW (thousands of k-blocks per tile against one epilogue) that this mode is
+//                  made for; a forward or dz unit is two vocabulary tiles.
 template <int MODE>
 struct Cfg {
   static constexpr bool PAIR = MODE != 0;                   // cta_group::2 on a 2-CTA cluster
   static constexpr int CL = PAIR ? 2 : 1;                   // CTAs per cluster
   static constexpr int NT = MODE == 2 ? 2 : 1;              // 256-column MMAs per k-step
   static constexpr int ACC_BUFS = MODE == 2 ? 1 : 2;        // accumulators in TMEM
+  // epilogue warps: 4 (one per TMEM lane quadrant), or 8 in mode 2 (two per quadrant, each
+  // reading one 256-column half of the single accumulator, which halves the time the next
+  // tile's MMAs wait for it)
+  static constexpr int EPI_WARPS = MODE == 2 ? 8 : 4;
+  static constexpr int THREADS = (2 + EPI_WARPS) * 32;
   static constexpr int STAGES = MODE == 1 ? 6 : 4;
   static constexpr uint32_t A_STAGE = BM * BK * 2;          // 16 KB
   static constexpr uint32_t B_HALF_ROWS = PAIR ? BN / 2 : BN;   // B rows per MMA staged here
@@ -285,9 +291,13 @@ __device__ void run_producer(const CUtensorMap* mapA, const CUtensorMap* mapB,
     // box of A / B this CTA loads.
     auto boxes = [&](int ti, int kbi, auto&& fa, auto&& fb) {
       if (ROLE == ROLE_FWD || ROLE == ROLE_DZ) {
-        const int vt = (ROLE == ROLE_FWD) ? n * kFwdTilesPerStrip + ti : a.vc0 / BN + n;
         fa(0u, mapA, kbi * BK, hrow);
-        fb(0u, mapB, kbi * BK, vt * BN + b_row0);
+#pragma unroll
+        for (int h = 0; h < NT; ++h) {   // wide pair: vocabulary tiles 2n and 2n+1
+          const int vt = (ROLE == ROLE_FWD) ? (n * NT + h) * kFwdTilesPerStrip + ti
+                                            : a.vc0 / BN + n * NT + h;
+          fb(h * C::B_HALF_STAGE, mapB, kbi * BK, vt * BN + b_row0);
+        }
       } else if (Dual<ROLE>::value) {
         // k-blocks 0 .. nk-1: policy (H, W); nk .. 2nk-1: reference (H_ref, W_ref)
         const int nk = dm.num_kb / 2;
@@ -544,6 +554,11 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
   const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
   const int32_t where = WHERE_GEMM_BASE + ROLE * 16 + 4;
   constexpr int NT = Cfg<MODE>::NT;   // 256-column halves of the accumulator tile
+  // columns of the accumulator tile this warp reads: all of them with 4 epilogue warps, one
+  // 256-column half (h = 0 for warps 2-5, 1 for warps 6-9) with 8
+  constexpr int CW = NT * BN / (Cfg<MODE>::EPI_WARPS / 4);
+  const int h = (warp - 2) / 4;
+  const int col0 = h * CW;
   uint32_t buf = 0, bphase = 0;
   uint32_t ob = 0;                    // dz staging buffer this warp fills next (TMA-store path)
   for (int u = sc.first; u < sc.num_units; u += sc.step) {
@@ -564,12 +579,12 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
       for (int t = 0; t < nacc; ++t) {
         if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
         tc_fence_after();
-        const int vbase = (n * kFwdTilesPerStrip + t) * BN;
-        for (int c = 0; c < BN / 32; ++c) {
+        const int vbase = (n * NT * kFwdTilesPerStrip + t) * BN + col0;
+        for (int c = 0; c < CW / 32; ++c) {
           const int v0 = vbase + c * 32;
           if (v0 >= a.V) break;  // uniform across the warp
           float x[32];
-          tmem_load_32cols(t_row + buf * BN + c * 32, x);
+          tmem_load_32cols(t_row + buf * BN + col0 + c * 32, x);
           const int nvalid = a.V - v0;
           if (nvalid < 32) {
 #pragma unroll
@@ -613,11 +628,12 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
           }
         }
         epi_release<MODE>(&acce[buf], lane, sc.rank);
-        buf ^= 1u;
-        if (buf == 0) bphase ^= 1u;
+        advance_buf<ROLE, MODE>(buf, bphase);
       }
-      if (m_ok)
-        a.partials[static_cast<long long>(n) * a.rows_cap + static_cast<long long>(m_load) * BM + r] =
+      const int strip = n * NT + h;   // this warp's strip of vocabulary columns
+      if (m_ok && strip < a.num_strips)
+        a.partials[static_cast<long long>(strip) * a.rows_cap +
+                   static_cast<long long>(m_load) * BM + r] =
             make_float4(rm, rs, ru, __int_as_float(ri));
       if (found) a.zy[pos] = zyv;
 
@@ -770,10 +786,11 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
       // dz of 32 consecutive columns of this row, bf16 pairs, from accumulator columns c*32..
+      // (c counts 32-column chunks from this warp's first column)
       auto dz_chunk = [&](int c, uint32_t (&pk)[16]) {
-        const int v0 = a.vc0 + n * BN + c * 32;
+        const int v0 = a.vc0 + n * NT * BN + col0 + c * 32;
         float x[32];
-        tmem_load_32cols(t_row + buf * BN + c * 32, x);
+        tmem_load_32cols(t_row + buf * BN + col0 + c * 32, x);
         if (act) {
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -818,11 +835,12 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
       } else {
         __nv_bfloat16* dst_row =
             a.dz + (static_cast<size_t>(m_load) * BM + r) * static_cast<size_t>(a.dz_pitch);
-        for (int c = 0; c < BN / 32; ++c) {
-          const int vloc = n * BN + c * 32;
+        for (int c = 0; c < CW / 32; ++c) {
+          const int vloc = n * NT * BN + col0 + c * 32;
           uint32_t pk[16];
           dz_chunk(c, pk);
-          if (!m_ok) continue;
+          // a wide unit's second tile may lie past the scratch row (odd tile count)
+          if (!m_ok || vloc >= a.dz_pitch) continue;
           uint4* dst = reinterpret_cast<uint4*>(dst_row + vloc);
 #pragma unroll
           for (int j = 0; j < 4; ++j)
@@ -830,8 +848,7 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
         }
       }
       epi_release<MODE>(&acce[buf], lane, sc.rank);
-      buf ^= 1u;
-      if (buf == 0) bphase ^= 1u;
+      advance_buf<ROLE, MODE>(buf, bphase);
 
     } else if (ROLE == ROLE_DH) {
       const int prow = a.row_pos[static_cast<long long>(m_load) * BM + r];  // position or -1
@@ -839,10 +856,10 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
       const long long pos = rv ? prow : 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
-      for (int c = 0; c < NT * BN / 32; ++c) {
-        const int col = n * NT * BN + c * 32;
+      for (int c = 0; c < CW / 32; ++c) {
+        const int col = n * NT * BN + col0 + c * 32;
         float x[32];
-        tmem_load_32cols(t_row + buf * BN + c * 32, x);
+        tmem_load_32cols(t_row + buf * BN + col0 + c * 32, x);
         if (!rv || col >= a.d) continue;   // columns past d (a partial last tile) hold zeros
         float* acc_row = a.dH_acc + (static_cast<size_t>(m_load) * BM + r) * a.d + col;
         if (a.dh_mode == 2 || a.dh_mode == 3) {
@@ -885,11 +902,11 @@ __device__ void run_epilogue_tiles(const GemmArgs& a, const Dims& dm, const Sche
       const bool empty_k = dm.num_kb == 0;
       if (!epi_wait(&accf[buf], bphase, abort_flag, a.hdr, where)) return;
       tc_fence_after();
-      float* dst_row = a.dW + static_cast<size_t>(a.vc0 + vrow) * a.d + n * NT * BN;
-      for (int c = 0; c < NT * BN / 32; ++c) {
+      float* dst_row = a.dW + static_cast<size_t>(a.vc0 + vrow) * a.d + n * NT * BN + col0;
+      for (int c = 0; c < CW / 32; ++c) {
         float x[32];
-        tmem_load_32cols(t_row + buf * BN + c * 32, x);
-        if (!rv || n * NT * BN + c * 32 >= a.d) continue;   // columns past d: a partial last tile
+        tmem_load_32cols(t_row + buf * BN + col0 + c * 32, x);
+        if (!rv || n * NT * BN + col0 + c * 32 >= a.d) continue;   // columns past d
         if (empty_k) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) x[j] = 0.f;
@@ -948,7 +965,7 @@ __device__ __forceinline__ void gemm_body(const CUtensorMap* mapA, const CUtenso
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], PAIR ? 8 : 4);  // epilogue warps of one or both CTAs
+      mbar_init(&acce[b], (PAIR ? 2 : 1) * C::EPI_WARPS);  // epilogue warps of one or both CTAs
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -1022,19 +1039,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
 // MODE 1 (256 x 256 tiles) or 2 (256 x 512 tiles) on CTA pairs.
 template <int ROLE, int MODE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Cfg<MODE>::THREADS, 1)
     tc_gemm_pair(const __grid_constant__ CUtensorMap mapA,
                  const __grid_constant__ CUtensorMap mapB, const __grid_constant__ GemmArgs args) {
   gemm_body<ROLE, MODE>(&mapA, &mapB, &mapA, &mapB, args);
 }
 
 template <class Kernel, class... Args>
-cudaError_t launch_with_smem(Kernel kernel, size_t smem, int grid, cudaStream_t st,
+cudaError_t launch_with_smem(Kernel kernel, size_t smem, int grid, int threads, cudaStream_t st,
                              Args&&... args) {
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  kernel<<<grid, NUM_THREADS, smem, st>>>(args...);
+  kernel<<<grid, threads, smem, st>>>(args...);
   return cudaGetLastError();
 }
 
@@ -1044,17 +1061,18 @@ cudaError_t launch_role(const CUtensorMap& mapA, const CUtensorMap& mapB, const 
                         const CUtensorMap& mapB2) {
   if constexpr (!Dual<ROLE>::value) {       // exact-KL roles: single-CTA tiles only
     if (mode == 1)
-      return launch_with_smem(tc_gemm_pair<ROLE, 1>, smem_bytes<ROLE, 1>(), grid, st, mapA, mapB,
-                              args);
-    if constexpr (ROLE == ROLE_DH || ROLE == ROLE_DW) {   // wide pair: the long-K roles only
+      return launch_with_smem(tc_gemm_pair<ROLE, 1>, smem_bytes<ROLE, 1>(), grid,
+                              Cfg<1>::THREADS, st, mapA, mapB, args);
+    // wide pair: a forward unit is two 256-column strips (one-tile strips only)
+    if constexpr (ROLE != ROLE_FWD || kFwdTilesPerStrip == 1) {
       if (mode == 2)
-        return launch_with_smem(tc_gemm_pair<ROLE, 2>, smem_bytes<ROLE, 2>(), grid, st, mapA,
-                                mapB, args);
+        return launch_with_smem(tc_gemm_pair<ROLE, 2>, smem_bytes<ROLE, 2>(), grid,
+                                Cfg<2>::THREADS, st, mapA, mapB, args);
     }
   }
   if (mode != 0) return cudaErrorInvalidValue;
-  return launch_with_smem(tc_gemm<ROLE>, smem_bytes<ROLE, 0>(), grid, st, mapA, mapB, mapA2,
-                          mapB2, args);
+  return launch_with_smem(tc_gemm<ROLE>, smem_bytes<ROLE, 0>(), grid, Cfg<0>::THREADS, st, mapA,
+                          mapB, mapA2, mapB2, args);
 }
 
 }  // namespace
@@ -1069,13 +1087,13 @@ int gemm_b_box_rows(int tile_mode) { return tile_mode == 0 ? BN : BN / 2; }
 
 namespace {
 template <typename Kernel>
-int query_active_clusters(Kernel kernel, size_t smem, int cl) {
+int query_active_clusters(Kernel kernel, size_t smem, int cl, int threads) {
   if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(smem)) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(cl), 1, 1);
-  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.blockDim = dim3(static_cast<unsigned>(threads), 1, 1);
   cfg.dynamicSmemBytes = smem;
   int n = 0;   // the kernels fix their cluster shape at compile time: no attribute here
   if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kernel), &cfg) !=
@@ -1101,8 +1119,10 @@ int gemm_max_clusters(int tile_mode) {
   int known = g_active_clusters[dev][tile_mode].load();
   if (known == 0) {
     int n = 0;
-    if (tile_mode == 1) n = query_active_clusters(tc_gemm_pair<ROLE_FWD, 1>, Cfg<1>::SMEM, cl);
-    if (tile_mode == 2) n = query_active_clusters(tc_gemm_pair<ROLE_DW, 2>, Cfg<2>::SMEM, cl);
+    if (tile_mode == 1)
+      n = query_active_clusters(tc_gemm_pair<ROLE_FWD, 1>, Cfg<1>::SMEM, cl, Cfg<1>::THREADS);
+    if (tile_mode == 2)
+      n = query_active_clusters(tc_gemm_pair<ROLE_DW, 2>, Cfg<2>::SMEM, cl, Cfg<2>::THREADS);
     known = n > 0 ? n : cap;   // a failed query falls back to one cluster per `cl` SMs
     g_active_clusters[dev][tile_mode].store(known);
   }

@@ -149,8 +149,7 @@ cudaError_t launch_f32_dw(const float* H, const float* W, const int32_t* tokens,
 
 // Tensor-core tile mode that GEMM role `role` (ROLE_*) runs in (the process-wide choice made
 // through grpo_set_tile_mode / grpo_set_role_tile_mode): 0 single CTA, 128 x 256 tiles
-// (cta_group::1); 1 CTA pair, 256 x 256 tiles (cta_group::2); 2 CTA pair, 256 x 512 tiles (DH
-// and DW only).
+// (cta_group::1); 1 CTA pair, 256 x 256 tiles (cta_group::2); 2 CTA pair, 256 x 512 tiles.
 int gemm_role_tile_mode(int role);
 
 // tcgen05 GEMM launches. `grid` = persistent CTAs.
@@ -169,7 +168,7 @@ int gemm_max_clusters(int tile_mode);
 // mode 2, 2 consecutive column tiles) per unit; never more CTAs than units need.
 int gemm_grid(long long row_tiles, long long col_tiles, int tile_mode);
 // tile_mode 1, 2: pair kernels; `grid` must be even and the K-major B map's box
-// gemm_b_box_rows(tile_mode) rows. Mode 2 is accepted for ROLE_DH and ROLE_DW only.
+// gemm_b_box_rows(tile_mode) rows. A forward unit in mode 2 needs one-tile strips.
 // mapA2 / mapB2 (H_ref, W_ref) are read by the KL roles only (single-CTA tiles).
 cudaError_t launch_gemm(int role, const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const GemmArgs& args, int grid, int tile_mode, cudaStream_t st,

@@ -484,7 +484,8 @@ ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW = 0, 1, 2, 3
 
 def grpo_set_tile_mode(mode: int):
     """Every GEMM role in one mode: 0 single-CTA 128 x 256 tiles, 1 CTA-pair 256 x 256 tiles
-    (cta_group::2); -1 (TILE_DEFAULT) restores each role's default."""
+    (cta_group::2), 2 CTA-pair 256 x 512 tiles; -1 (TILE_DEFAULT) restores each role's
+    default."""
     _check(_lib().grpo_set_tile_mode(int(mode)), "grpo_set_tile_mode")
 
 
@@ -494,8 +495,8 @@ def grpo_get_tile_mode() -> int:
 
 
 def grpo_set_role_tile_mode(role: int, mode: int):
-    """Tile mode of one GEMM role (ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW): 0, 1, or for ROLE_DH and
-    ROLE_DW also 2 (CTA-pair 256 x 512 tiles); -1 restores the role's default."""
+    """Tile mode of one GEMM role (ROLE_FWD, ROLE_DZ, ROLE_DH, ROLE_DW): 0, 1 or 2; -1 restores
+    the role's default."""
     _check(_lib().grpo_set_role_tile_mode(int(role), int(mode)), "grpo_set_role_tile_mode")
 
 

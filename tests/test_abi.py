@@ -72,16 +72,16 @@ def test_host_validation_rejects_before_launch(lib):
 
 
 def test_process_wide_settings_validate_and_round_trip(lib):
-    """Host-only setters (no GPU work): tile modes 0 and 1 accepted for every role at once and
-    read back, others refused (mode 2 is per-role only); the progress window refuses a negative
+    """Host-only setters (no GPU work): tile modes 0, 1 and 2 accepted for every role at once
+    and read back, others refused; the progress window refuses a negative
     lag and a checkpoint with lag 0, and takes negative checkpoint spacings (in work units); the
     CTA-pair switch maps to tile modes 1 / 0."""
     try:
-        for mode in (0, 1):
+        for mode in (0, 2, 1):
             assert lib.grpo_set_tile_mode(mode) == 0
             assert lib.grpo_get_tile_mode() == mode
             assert [lib.grpo_get_role_tile_mode(r) for r in range(4)] == [mode] * 4
-        for bad in (-2, 2, 3, 4, 5, 1 << 20):
+        for bad in (-2, 3, 4, 5, 1 << 20):
             assert lib.grpo_set_tile_mode(bad) == -1
             assert lib.grpo_get_tile_mode() == 1          # unchanged by a refused call
         assert lib.grpo_set_cta_pair(0) == 0 and lib.grpo_get_tile_mode() == 0
@@ -101,15 +101,14 @@ def test_process_wide_settings_validate_and_round_trip(lib):
 def test_role_tile_modes_defaults_overrides_and_refusals(lib):
     """Per-role tile modes (host-only): the library starts with its per-role defaults (forward
     and dz 0, dH and dW 2; the shared mode then reads -1), an override changes its own role
-    only, -1 restores defaults, the wide pair (2) is refused for the forward and dz roles, and
-    bad roles or modes are refused without changing anything."""
+    only, -1 restores defaults, and bad roles or modes are refused without changing anything."""
     try:
         assert lib.grpo_set_tile_mode(-1) == 0
         assert [lib.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 0, 2, 2]
         assert lib.grpo_get_tile_mode() == -1
         assert lib.grpo_set_role_tile_mode(1, 1) == 0
         assert [lib.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 1, 2, 2]
-        for role, mode in ((-1, 0), (4, 0), (0, -2), (1, 3), (0, 2), (1, 2), (2, 3), (3, 4)):
+        for role, mode in ((-1, 0), (4, 0), (0, -2), (1, 3), (2, 3), (3, 4)):
             assert lib.grpo_set_role_tile_mode(role, mode) == -1
         assert [lib.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 1, 2, 2]
         assert lib.grpo_get_role_tile_mode(4) == -1 and lib.grpo_get_role_tile_mode(-1) == -1

@@ -76,14 +76,16 @@ def test_partial_hidden_tile_chunked_backward_and_every_tile_mode():
     columns, and 2600 / 128 = 21 vocabulary row tiles of dW (odd: the second CTA of the last
     pair stages a copy). A 3-chunk backward (V = 2600 in chunks of 1024) accumulates dH across
     chunks through the partial tile in every mode. Every mode meets the parity bar; dH and dW of
-    mode 2 are bitwise equal to mode 1's on the same dz."""
+    mode 2 are bitwise equal to mode 1's on the same dz, and with every role in mode 2 (forward
+and dz units of two vocabulary tiles; V = 2600 has 11 tiles, so the last unit's second tile
+lies past the vocabulary) every output is bitwise equal to mode 1's."""
     from paper_2510_17158_gb300 import grpo as G
     b = make_batch_numpy(W_("d576_v2600", 1, (4,), 160, 40, 160, 576, 2600))
     old, ref = oracle_inputs(b)
     o = run_oracle(b, old, ref, 0.2, 0.2, 0.04)
     outs = {}
     try:
-        for modes in ((0, 0, 0, 0), (1, 1, 1, 1), (1, 1, 2, 2), (0, 0, 2, 2)):
+        for modes in ((0, 0, 0, 0), (1, 1, 1, 1), (1, 1, 2, 2), (0, 0, 2, 2), (2, 2, 2, 2)):
             for role, m in enumerate(modes):
                 G.grpo_set_role_tile_mode(role, m)
             outs[modes] = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
@@ -94,3 +96,5 @@ def test_partial_hidden_tile_chunked_backward_and_every_tile_mode():
         G.grpo_set_tile_mode(G.TILE_DEFAULT)
     for k in ("dH", "dW"):
         assert torch.equal(outs[(1, 1, 2, 2)][k], outs[(1, 1, 1, 1)][k]), k
+    for k in ("logp", "lse", "entropy", "argmax", "dH", "dW"):   # the same M = 256 MMAs
+        assert torch.equal(outs[(2, 2, 2, 2)][k], outs[(1, 1, 1, 1)][k]), k

@@ -138,7 +138,7 @@ def test_tile_modes_match_oracle(name):
     assert [G.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 0, 2, 2]
     assert G.grpo_get_tile_mode() == G.TILE_DEFAULT
     try:
-        for modes in ((0, 0, 0, 0), (1, 1, 1, 1), (0, 0, 2, 2), (1, 1, 2, 2)):
+        for modes in ((0, 0, 0, 0), (1, 1, 1, 1), (0, 0, 2, 2), (1, 1, 2, 2), (2, 2, 2, 2)):
             _set_roles(G, modes)
             g = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
             print("modes", modes, compare(b, g, o))
@@ -149,10 +149,12 @@ def test_tile_modes_match_oracle(name):
 @pytest.mark.parametrize("name", ["d2048_v32k"])
 def test_tile_mode_mixes_bitwise_relations(name):
     """Each GEMM role runs in its own tile mode (grpo_set_role_tile_mode). Results that must be
-    bitwise equal: the forward statistics and the loss whenever the forward role's mode is the
-    same (they do not depend on the backward roles), and dH, dW between modes 1 and 2 of the
-    backward roles on the same dz (both issue the same M = 256, N = 256 MMAs for every output
-    element, in the same k order). Mode 0 against the pair modes agrees within the parity bar."""
+    bitwise equal: the forward statistics and the loss between the pair modes 1 and 2 of the
+    forward role, and whenever the forward role's mode is the same (they do not depend on the
+    backward roles); dz and hence dH, dW between modes 1 and 2 of the dz role; dH, dW between
+    modes 1 and 2 of the backward roles on the same dz (modes 1 and 2 issue the same M = 256,
+    N = 256 MMAs for every output element, in the same k order). Mode 0 against the pair modes
+    agrees within the parity bar."""
     from paper_2510_17158_gb300 import grpo as G
     b = _batch(name)
     old, ref = oracle_inputs(b)
@@ -160,19 +162,19 @@ def test_tile_mode_mixes_bitwise_relations(name):
     outs = {}
     try:
         for modes in ((0, 0, 0, 0), (0, 0, 1, 1), (0, 0, 2, 2), (0, 0, 1, 2), (0, 0, 2, 1),
-                      (1, 1, 1, 1), (1, 1, 2, 2), (0, 1, 2, 2)):
+                      (1, 1, 1, 1), (1, 1, 2, 2), (0, 1, 2, 2), (2, 2, 2, 2), (2, 1, 1, 2)):
             _set_roles(G, modes)
             outs[modes] = run_gpu(b, old, ref, 0.2, 0.2, 0.04)
             print("roles", modes, compare(b, outs[modes], o))
     finally:
         G.grpo_set_tile_mode(G.TILE_DEFAULT)
-    for modes, g in outs.items():
+    for modes, g in outs.items():   # forward in mode 1 or 2: the same M = 256, N = 256 MMAs
         ref_fwd = outs[(0, 0, 0, 0)] if modes[0] == 0 else outs[(1, 1, 1, 1)]
         for k in MODE_KEYS_FWD:
             assert torch.equal(g[k], ref_fwd[k]), (modes, k)
         assert g["loss"] == ref_fwd["loss"], modes
     same_dz = [((0, 0, 1, 1), (0, 0, 2, 2), (0, 0, 1, 2), (0, 0, 2, 1)),
-               ((1, 1, 1, 1), (1, 1, 2, 2))]
+               ((1, 1, 1, 1), (1, 1, 2, 2), (2, 2, 2, 2), (2, 1, 1, 2))]
     for group in same_dz:
         for modes in group[1:]:
             for k in ("dH", "dW"):
@@ -182,12 +184,12 @@ def test_tile_mode_mixes_bitwise_relations(name):
 def test_tile_mode_rejects_unknown_modes():
     from paper_2510_17158_gb300 import grpo as G
     prev = G.grpo_get_tile_mode()
-    for bad in (-2, 2, 5):
+    for bad in (-2, 3, 5):
         with pytest.raises(G.GrpoError):
             G.grpo_set_tile_mode(bad)
     assert G.grpo_get_tile_mode() == prev
     with pytest.raises(G.GrpoError):
-        G.grpo_set_role_tile_mode(G.ROLE_FWD, G.TILE_CTA_PAIR_WIDE)
+        G.grpo_set_role_tile_mode(G.ROLE_FWD, 3)
 
 
 def test_chunked_backward_full_vocabulary_partial_last_chunk():
