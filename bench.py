@@ -470,8 +470,8 @@ def run_gpu(args):
                    "d": d, "V": V, "eps": w.eps, "beta": w.beta, "scored_tokens_per_rank": N_v,
                    "vocab_chunk": args.vocab_chunk or "whole vocabulary",
                    "tiles": tiles_desc(G),
-                   "gemm_window": ("library default (dH, dW: checkpoint at every work unit, "
-                                   "lag 1)" if win is None else "off" if win[0] == 0 else
+                   "gemm_window": ("library default (dH, dW: a barrier every 256 k-blocks)"
+                                   if win is None else "off" if win[0] == 0 else
                                    f"{win[0]} k-blocks, lag {win[1]} checkpoints" if win[0] > 0
                                    else f"every {-win[0]} work unit(s), lag {win[1]}"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (

@@ -303,9 +303,11 @@ int grpo_get_role_tile_mode(int32_t role);
  * to hit L2 (CTAs that share a tile otherwise drift apart over successive long-K units and
  * re-read their operands from HBM). Checkpoints fall every `check_kblocks` k-blocks of 64
  * (check_kblocks > 0) or, for check_kblocks < 0, at the start of every (-check_kblocks)-th work
- * unit (an output tile): with lag 1 a barrier between the waves of units. Default (-1, 1).
- * Results do not depend on it. check_kblocks == 0 turns it off. Returns GRPO_ERR_INVALID_ARG
- * for a negative lag or for check_kblocks != 0 with lag == 0. */
+ * unit (an output tile): with lag 1 a barrier between the waves of units. Default
+ * (GRPO_GEMM_WINDOW_DEFAULT_CHECK, GRPO_GEMM_WINDOW_DEFAULT_LAG) = (256, 1): a barrier every 256
+ * k-blocks. Results do not depend on it. check_kblocks == 0 turns it off. Returns
+ * GRPO_ERR_INVALID_ARG for a negative lag or for check_kblocks != 0 with lag == 0. */
+enum { GRPO_GEMM_WINDOW_DEFAULT_CHECK = 256, GRPO_GEMM_WINDOW_DEFAULT_LAG = 1 };
 int grpo_set_gemm_window(int32_t check_kblocks, int32_t lag);
 
 #ifdef __cplusplus

@@ -40,11 +40,11 @@ constexpr int kRoleDefault[4] = {GRPO_TILE_SINGLE, GRPO_TILE_SINGLE, GRPO_TILE_C
                                  GRPO_TILE_CTA_PAIR_WIDE};
 std::atomic<int> g_role_mode[4] = {{kRoleDefault[0]}, {kRoleDefault[1]}, {kRoleDefault[2]},
                                    {kRoleDefault[3]}};
-// GEMM progress window of the long-K roles (checkpoint spacing, lag): by default a checkpoint at
-// the start of every dH / dW work unit with lag 1, i.e. a barrier between the waves of units,
-// which keeps the CTA pairs that share a dz or W tile within the L2's reuse window (dH and dW
-// 296 -> 274-277 ms at 2 x 16 completions, T = 16384, d = 5120, V = 151936).
-std::atomic<int> g_win_check{-1}, g_win_lag{1};
+// GEMM progress window of the long-K roles (checkpoint spacing, lag): by default a barrier every
+// 256 k-blocks of dH and dW (lag 1), which keeps the CTA pairs that share a dz or W tile within
+// the L2's reuse window (dH and dW 296 -> 265-267 ms at 2 x 16 completions, T = 16384,
+// d = 5120, V = 151936; a barrier at every work unit's start: 267-268 ms, 10 % more DRAM bytes).
+std::atomic<int> g_win_check{GRPO_GEMM_WINDOW_DEFAULT_CHECK}, g_win_lag{GRPO_GEMM_WINDOW_DEFAULT_LAG};
 std::atomic<long long> g_launches[GRPO_K_COUNT];
 std::vector<EventPair> g_pending[GRPO_K_COUNT];
 double g_total_ms[GRPO_K_COUNT];

@@ -37,8 +37,10 @@ constexpr int NUM_THREADS = 192;          // 6 warps (modes 0, 1); mode 2: Cfg<2
 // Raster groups: row tiles that consecutive work units walk before moving to the next column
 // unit, per role. Measured on a power-capped GB300 at 2 x 16 completions, T = 16384, d = 5120,
 // V = 151936 (the GEMM's time against the neighbouring values): forward 32 (16: +0-2 %,
-// 8: +7 %), dz recompute 32 (16: +1.5 %, 64: +15 %), dH and dW 64 (16: +7 %, 32: +2 %, 128:
-// +0.5 %, measured without the progress window).
+// 48: +8 %, 64: +14 %: the group's H rows no longer stay in L2), dz recompute 32 (16: +1.5 %,
+// 48: +9 %, 64: +12 %), dH and dW 32 (24, 48: +0.5-1 %; 64: +1 %, with 20-24 % more DRAM
+// bytes). A wave of 76 CTA-pair units covers g/2 row units x 152/g column units, so larger
+// groups re-read the row operand (dz) more often and smaller ones the column operand (W, Hp).
 #ifndef GRPO_GROUP_M_FWD
 #define GRPO_GROUP_M_FWD 32
 #endif
@@ -46,10 +48,10 @@ constexpr int NUM_THREADS = 192;          // 6 warps (modes 0, 1); mode 2: Cfg<2
 #define GRPO_GROUP_M_DZ 32
 #endif
 #ifndef GRPO_GROUP_M_DH
-#define GRPO_GROUP_M_DH 64
+#define GRPO_GROUP_M_DH 32
 #endif
 #ifndef GRPO_GROUP_M_DW
-#define GRPO_GROUP_M_DW 64
+#define GRPO_GROUP_M_DW 32
 #endif
 template <int ROLE>
 constexpr int group_rows() {

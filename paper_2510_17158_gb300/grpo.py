@@ -21,6 +21,7 @@ HEADER_PATH = os.path.join(os.path.dirname(_HERE), "include", "grpo.h")
 
 GRPO_F32, GRPO_BF16 = 0, 1
 STATIC_SCRATCH_BYTES = 64 << 20      # GRPO_STATIC_SCRATCH_BYTES of include/grpo.h
+GEMM_WINDOW_DEFAULT = (256, 1)       # GRPO_GEMM_WINDOW_DEFAULT_{CHECK,LAG} of include/grpo.h
 STD_MODES = {"unbiased": 0, "population": 1}
 AGG_MODES = {"seq_mean": 0, "token_mean": 1}
 STATUS_NAMES = {0: "GRPO_OK", -1: "GRPO_ERR_INVALID_ARG", -2: "GRPO_ERR_UNSUPPORTED",
@@ -508,8 +509,9 @@ def grpo_get_role_tile_mode(role: int) -> int:
 
 
 def grpo_set_gemm_window(check_kblocks: int, lag: int):
-    """GEMM progress window: producers stay within `lag` checkpoints of `check_kblocks` k-blocks
-    of the launch's average (0 turns it off, the default)."""
+    """Progress window of the dH and dW GEMMs: producers stay within `lag` checkpoints of the
+    launch's average, a checkpoint every `check_kblocks` k-blocks (< 0: at the start of every
+    (-check_kblocks)-th work unit; 0 turns it off). Default: GEMM_WINDOW_DEFAULT."""
     _check(_lib().grpo_set_gemm_window(int(check_kblocks), int(lag)), "grpo_set_gemm_window")
 
 

@@ -95,7 +95,7 @@ def test_process_wide_settings_validate_and_round_trip(lib):
     assert lib.grpo_set_gemm_window(-1, 1) == 0      # checkpoints at every unit start
     assert lib.grpo_set_gemm_window(-2, 2) == 0
     assert lib.grpo_set_gemm_window(0, 0) == 0
-    assert lib.grpo_set_gemm_window(-1, 1) == 0      # back to the library's default
+    assert lib.grpo_set_gemm_window(*G.GEMM_WINDOW_DEFAULT) == 0   # back to the library's default
 
 
 def test_role_tile_modes_defaults_overrides_and_refusals(lib):
@@ -122,3 +122,15 @@ def test_role_tile_modes_defaults_overrides_and_refusals(lib):
         assert [lib.grpo_get_role_tile_mode(r) for r in range(4)] == [0, 0, 1, 1]
     finally:
         lib.grpo_set_tile_mode(-1)
+
+
+def test_python_constants_match_the_header():
+    """The binding's copies of the header's constants: the static scratch size and the progress
+    window's default, read from include/grpo.h as text."""
+    import re
+    text = open(G.HEADER_PATH).read()
+    m = re.search(r"#define GRPO_STATIC_SCRATCH_BYTES \((\d+)u \* (\d+)u \* (\d+)u\)", text)
+    assert m and int(m[1]) * int(m[2]) * int(m[3]) == G.STATIC_SCRATCH_BYTES
+    check = int(re.search(r"GRPO_GEMM_WINDOW_DEFAULT_CHECK = (-?\d+)", text)[1])
+    lag = int(re.search(r"GRPO_GEMM_WINDOW_DEFAULT_LAG = (\d+)", text)[1])
+    assert (check, lag) == G.GEMM_WINDOW_DEFAULT

@@ -210,15 +210,16 @@ def test_chunked_backward_full_vocabulary_partial_last_chunk():
 def test_progress_window_changes_nothing_and_resets_its_counters():
     """The progress window of the dH and dW GEMMs only delays TMA issue: outputs with it off, at
     16 k-blocks with lag 4, at a tight setting (1 k-block, lag 1, so that the producers wait at
-    every k-block) and with checkpoints at every work unit's start (-1, lag 1: a barrier between
-    waves of units, the default) are bitwise equal, and the last CTA of every launch resets the
-    window's counters in the workspace header (arrivals at byte 24, CTAs left at byte 32) to 0."""
+    every k-block), with checkpoints at every work unit's start (-1, lag 1: a barrier between
+    waves of units) and at the default (a barrier every 256 k-blocks) are bitwise equal, and the
+    last CTA of every launch resets the window's counters in the workspace header (arrivals at
+    byte 24, CTAs left at byte 32) to 0."""
     from paper_2510_17158_gb300 import grpo as G
     b = _batch("d4096_v152k")
     old, ref = oracle_inputs(b)
     outs = []
     try:
-        for check, lag in ((0, 0), (16, 4), (1, 1), (-1, 1)):
+        for check, lag in ((0, 0), (16, 4), (1, 1), (-1, 1), G.GEMM_WINDOW_DEFAULT):
             G.grpo_set_gemm_window(check, lag)
             outs.append(run_gpu(b, old, ref, 0.2, 0.2, 0.04))
             dev = torch.device("cuda")
@@ -235,7 +236,7 @@ def test_progress_window_changes_nothing_and_resets_its_counters():
             assert int(hdr[24:32].view(np.uint64)[0]) == 0
             assert int(hdr[32:36].view(np.uint32)[0]) == 0
     finally:
-        G.grpo_set_gemm_window(-1, 1)
+        G.grpo_set_gemm_window(*G.GEMM_WINDOW_DEFAULT)
     for g in outs[1:]:
         for k in ("logp", "lse", "entropy", "argmax", "valid_count", "dH", "dW"):
             assert torch.equal(g[k], outs[0][k]), k
