@@ -534,7 +534,7 @@ def main():
                     help="progress window of the dH and dW GEMMs CHECK,LAG: producers stay within "
                          "LAG checkpoints of the launch's average; checkpoints every CHECK "
                          "k-blocks, or at every -CHECK-th work unit for CHECK < 0 (write "
-                         "--gemm-window=-1,1); '0,0' = off; default: the library's (-1,1)")
+                         "--gemm-window=-1,1); '0,0' = off; default: the library's (256,1)")
     ap.add_argument("--graph", action="store_true",
                     help="capture one step in a CUDA graph and time its replays (per-kernel "
                          "timing and launch counts then come from the capture, not the replays)")
