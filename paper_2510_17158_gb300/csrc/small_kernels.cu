@@ -241,6 +241,26 @@ struct StripMerge {
   float rescale = 1.f;   // factor the running sums were multiplied by in the last add()
 };
 
+// Strips are read in batches of kMergeBatch independent loads before they are merged, in the
+// same vocabulary order: each thread then keeps that many loads in flight, which is what keeps
+// HBM busy when there are few positions (one load at a time leaves small batches latency bound).
+constexpr int kMergeBatch = 8;
+
+__device__ __forceinline__ void merge_strips(const float4* __restrict__ partials,
+                                             long long rows_cap, int num_strips, long long row,
+                                             StripMerge& mg) {
+  int j = 0;
+  for (; j + kMergeBatch <= num_strips; j += kMergeBatch) {
+    float4 p[kMergeBatch];
+#pragma unroll
+    for (int k = 0; k < kMergeBatch; ++k)
+      p[k] = partials[static_cast<long long>(j + k) * rows_cap + row];
+#pragma unroll
+    for (int k = 0; k < kMergeBatch; ++k) mg.add(p[k]);
+  }
+  for (; j < num_strips; ++j) mg.add(partials[static_cast<long long>(j) * rows_cap + row]);
+}
+
 __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_cap,
                             int num_strips, const float* __restrict__ zy,
                             const int32_t* __restrict__ pos_row,
@@ -259,7 +279,7 @@ __global__ void k_fwd_merge(const float4* __restrict__ partials, long long rows_
   }
   const long long row = pos_row[pos];   // packed row of this scored position
   StripMerge mg;
-  for (int j = 0; j < num_strips; ++j) mg.add(partials[static_cast<long long>(j) * rows_cap + row]);
+  merge_strips(partials, rows_cap, num_strips, row, mg);
   const float M = mg.M, Ssum = mg.S, U = mg.U;
   const int idx = mg.idx;
   const float lse = M + logf(Ssum);
@@ -304,9 +324,7 @@ __global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
   StripMerge mg;                        // policy: (m, s, u, argmax)
   float C = 0.f;                        // sum e^{z-M} z_ref in the policy's frame
   float Mr = -INFINITY, Sr = 0.f;       // reference: running max and sum e^{z_ref - Mr}
-  for (int j = 0; j < num_strips; ++j) {
-    const float4 p = partials[static_cast<long long>(j) * rows_cap + row];
-    const float4 q = partials2[static_cast<long long>(j) * rows_cap + row];
+  auto add = [&](const float4 p, const float4 q) {
     const float sc = mg.add(p);
     C = fmaf(C, mg.rescale, q.x * sc);
     if (q.y > Mr) {
@@ -315,7 +333,21 @@ __global__ void k_fwd_merge_kl(const float4* __restrict__ partials,
     } else {
       Sr = fmaf(q.z, ex2_approx((q.y - Mr) * kLog2e), Sr);
     }
+  };
+  int j = 0;
+  for (; j + kMergeBatch <= num_strips; j += kMergeBatch) {   // batched loads, as merge_strips
+    float4 p[kMergeBatch], q[kMergeBatch];
+#pragma unroll
+    for (int k = 0; k < kMergeBatch; ++k) {
+      p[k] = partials[static_cast<long long>(j + k) * rows_cap + row];
+      q[k] = partials2[static_cast<long long>(j + k) * rows_cap + row];
+    }
+#pragma unroll
+    for (int k = 0; k < kMergeBatch; ++k) add(p[k], q[k]);
   }
+  for (; j < num_strips; ++j)
+    add(partials[static_cast<long long>(j) * rows_cap + row],
+        partials2[static_cast<long long>(j) * rows_cap + row]);
   const float M = mg.M, Ssum = mg.S, U = mg.U;
   const int idx = mg.idx;
   const float lse = M + logf(Ssum);
@@ -467,7 +499,7 @@ __global__ void k_shard_stats(const float4* __restrict__ partials, long long row
   }
   const long long row = pos_row[pos];   // packed row of this scored position
   StripMerge mg;
-  for (int j = 0; j < num_strips; ++j) mg.add(partials[static_cast<long long>(j) * rows_cap + row]);
+  merge_strips(partials, rows_cap, num_strips, row, mg);
   stats[pos] = make_float4(mg.M, mg.S, mg.U, __int_as_float(mg.idx + v_offset));
   const int yl = tokens[pos] - v_offset;
   zy_out[pos] = (yl >= 0 && yl < V_shard) ? zy_ws[pos] : -INFINITY;
