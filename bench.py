@@ -95,6 +95,17 @@ def barrier(ws):
         dist.barrier()
 
 
+def dp_exchange(bwd_out: dict, ws: int):
+    """The data-parallel step's one exchange: every rank scored its own whole groups with the
+    global normaliser, so the summed loss and dW are the single-process ones; dH rows stay with
+    the rank that owns them. Issued on the current stream, inside the timed step."""
+    if ws > 1:
+        import torch.distributed as dist
+        dist.all_reduce(bwd_out["dW"], op=dist.ReduceOp.SUM)
+        dist.all_reduce(bwd_out["loss"], op=dist.ReduceOp.SUM)
+    return bwd_out
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle-reason samples every 200 ms while the timed region runs."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -342,6 +353,15 @@ def run_gpu(args):
     bwd_out = {"loss": torch.empty(1, device=device), "dH": torch.empty_like(b.H),
                "dW": torch.empty((V, d), dtype=torch.float32, device=device)}
     adv = torch.empty(S, device=device)
+    # loss normaliser over all ranks (Eq. 1's expectation over every rank's sequences, or every
+    # scored token for the distillation loss); 0 = this batch's own count
+    norm = 0.0
+    if ws_n > 1:
+        from paper_2510_17158_gb300 import dp
+        norm = dp.global_norm("token_mean" if args.path == "sft" else "seq_mean", S, N_v,
+                              lambda x: dist_sum(x, ws_n, device))
+        if args.graph:
+            raise SystemExit("--graph with more than one rank: the dW all-reduce is not captured")
     torch.cuda.synchronize()
     gen_s = time.time() - t_gen
 
@@ -349,19 +369,22 @@ def run_gpu(args):
         if args.path == "grpo-exact-kl":   # Eq. 1's KL over the whole vocabulary
             G.group_advantages(rewards, go, ws, adv_out=adv)
             f = G.grpo_score_fwd_kl(H, W, H_ref, W_ref, tok, mask, ws, out=fwd_out)
-            return G.grpo_loss_bwd_kl(H, W, H_ref, W_ref, tok, mask, f, old_, adv, ws,
-                                      eps_low=w.eps, eps_high=w.eps, beta=w.beta, out=bwd_out)
-        if args.path == "sft":       # distillation step (Sec. 6.2): no advantages, no ratio
+            o = G.grpo_loss_bwd_kl(H, W, H_ref, W_ref, tok, mask, f, old_, adv, ws,
+                                   eps_low=w.eps, eps_high=w.eps, beta=w.beta, norm=norm,
+                                   out=bwd_out)
+        elif args.path == "sft":     # distillation step (Sec. 6.2): no advantages, no ratio
             f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
-            return G.grpo_sft_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], f["valid_count"],
-                                       ws, out=bwd_out)
-        G.group_advantages(rewards, go, ws, adv_out=adv)
-        f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
-        if w.beta == 0.0:          # no KL term: the reference log-probs are not read
-            ref_ = None
-        return G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_, ref_, adv,
-                               f["valid_count"], ws, eps_low=w.eps, eps_high=w.eps, beta=w.beta,
-                               out=bwd_out)
+            o = G.grpo_sft_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], f["valid_count"],
+                                    ws, norm=norm, out=bwd_out)
+        else:
+            G.group_advantages(rewards, go, ws, adv_out=adv)
+            f = G.grpo_score_fwd(H, W, tok, mask, ws, out=fwd_out)
+            if w.beta == 0.0:      # no KL term: the reference log-probs are not read
+                ref_ = None
+            o = G.grpo_loss_bwd(H, W, tok, mask, f["logp"], f["lse"], old_, ref_, adv,
+                                f["valid_count"], ws, eps_low=w.eps, eps_high=w.eps,
+                                beta=w.beta, norm=norm, out=bwd_out)
+        return dp_exchange(o, ws_n)
 
     dev_args = (b.H, b.W, b.tokens, b.mask, b.rewards, b.group_offsets, old, ref)
     for _ in range(args.warmup):
@@ -476,7 +499,9 @@ def run_gpu(args):
                                    else f"every {-win[0]} work unit(s), lag {win[1]}"),
                    "l2": "inputs larger than L2 (H %.2f GB, W %.2f GB resident in HBM)" % (
                        b.H.numel() * 2 / 1e9, b.W.numel() * 2 / 1e9),
-                   "parallelism": f"dp{ws_n} (independent groups per GPU)",
+                   "parallelism": (f"dp{ws_n} (whole groups per GPU, global loss normaliser; dW "
+                                   "and loss all-reduced over NCCL every step)" if ws_n > 1 else
+                                   "dp1"),
                    "cuda_graph": bool(args.graph)},
         "tflops_alg": round(alg_tflops, 1),
         "frac_of_bf16_peak": round(alg_tflops / pk["bf16"], 4),

@@ -1,6 +1,7 @@
 """Data-parallel sharding over whole groups, checked with two gloo ranks on CPU against the
 single-process oracle: summed losses and dW, and each shard's dH rows, equal the whole-batch
-result when every rank uses the global normaliser."""
+result when every rank uses the global normaliser. The sums go through bench.py's per-step
+exchange (`dp_exchange`), the one its multi-GPU runs issue over NCCL."""
 import os
 import socket
 
@@ -10,6 +11,7 @@ import torch
 import torch.distributed as dist
 import torch.multiprocessing as mp
 
+import bench
 import oracle
 from paper_2510_17158_gb300.dp import global_norm, shard_groups
 from paper_2510_17158_gb300.synthetic import Workload, make_batch_numpy
@@ -49,11 +51,11 @@ def _worker(rank, port, agg, q):
     norm = global_norm(agg, hi - lo, int((mask != 0).sum()), allsum)
     o = oracle.grpo_step(H[lo:hi], W, b.tokens.numpy()[lo:hi], mask, b.rewards.numpy()[lo:hi],
                          go_local, old[lo:hi], ref[lo:hi], 0.2, 0.2, 0.04, agg=agg, norm=norm)
-    loss = torch.tensor([o["loss"]], dtype=torch.float64)
-    dW = torch.from_numpy(o["dW"].copy())
-    dist.all_reduce(loss)
-    dist.all_reduce(dW)
-    q.put((rank, lo, hi, float(loss.item()), dW.numpy(), o["dH"]))
+    dH = torch.from_numpy(o["dH"].copy())
+    out = bench.dp_exchange({"loss": torch.tensor([o["loss"]], dtype=torch.float64),
+                             "dW": torch.from_numpy(o["dW"].copy()), "dH": dH.clone()}, WORLD)
+    assert torch.equal(out["dH"], dH)   # dH rows stay with the rank that owns them
+    q.put((rank, lo, hi, float(out["loss"].item()), out["dW"].numpy(), o["dH"]))
     dist.destroy_process_group()
 
 
@@ -92,3 +94,4 @@ def test_shard_groups_covers_whole_groups():
     assert [p[:2] for p in parts] == [(0, 4), (4, 12), (12, 28)]
     for lo, hi, local in parts:
         assert local[0] == 0 and local[-1] == hi - lo
+
