@@ -338,7 +338,7 @@ def run_gpu(args):
     S, T, d, V = w.S, w.T, w.d, w.V
     N_v = int(b.mask.sum().item())
     ws = G.Workspace.for_problem(S, T, d, V, b.H.dtype, vocab_chunk=args.vocab_chunk,
-                                 device=device)
+                                 device=device, kl=args.path == "grpo-exact-kl")
     stream = torch.cuda.current_stream(device)
     # old / ref log-probs: the policy's own log-prob (a scoring pass) plus the workload's noise
     f0 = G.grpo_score_fwd(b.H, b.W, b.tokens, b.mask, ws)

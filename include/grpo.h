@@ -60,9 +60,14 @@ typedef enum { GRPO_AGG_SEQ_MEAN = 0, GRPO_AGG_TOKEN_MEAN = 1 } grpo_agg;
 /* Bytes of workspace needed for a problem of this shape. `vocab_chunk` is how many vocabulary
  * columns of dL/dz the backward keeps at once (rounded up to a multiple of 256); 0 = the whole
  * vocabulary in one chunk (fastest; S*ceil(T/128)*128*V*2 bytes of scratch). Returns 0 for
- * invalid shapes. The workspace must be 256-byte aligned. */
+ * invalid shapes. The workspace must be 256-byte aligned. The exact-KL entry points
+ * (grpo_score_fwd_kl, grpo_loss_bwd_kl) need grpo_workspace_bytes_kl instead, which adds the
+ * reference model's packed hidden states and forward statistics (bf16 only; 0 for f32); a
+ * workspace of that size serves every entry point. */
 size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
                             int32_t vocab_chunk);
+size_t grpo_workspace_bytes_kl(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                               int32_t vocab_chunk);
 
 /* Clears the workspace's status word. Call once after allocating a workspace. */
 int grpo_workspace_init(void* workspace, size_t workspace_bytes, grpo_stream_t stream);
@@ -168,7 +173,8 @@ int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new
  *   KL_t = sum_v p_tv (log p_tv - log q_tv),  p = softmax(W h_t),  q = softmax(W_ref h_ref_t).
  * grpo_score_fwd_kl computes grpo_score_fwd's outputs plus lse_ref [S,T] and kl [S,T] (0 at
  * unscored positions); both products stream through one tensor-core tile per 128 x 256 block,
- * the logits of neither model reach memory. H_ref [S,T,d], W_ref [V,d] bf16. */
+ * the logits of neither model reach memory. H_ref [S,T,d], W_ref [V,d] bf16. Workspace:
+ * grpo_workspace_bytes_kl (a smaller one returns GRPO_ERR_WORKSPACE). */
 int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
                       int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
                       int32_t T, int32_t d, int32_t V, float* logp, float* lse, float* entropy,
@@ -178,7 +184,8 @@ int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const voi
 /* grpo_loss_bwd with the exact KL: l_t = -surr_t + beta KL_t (the clipped surrogate as in
  * grpo_loss_bwd), and dz_t = g_t (onehot(y_t) - p_t) + beta w_t p_t (log p_t - log q_t - KL_t)
  * from both recomputed products; dH, dW as in grpo_loss_bwd (nothing flows to the frozen
- * reference). logp, lse, lse_ref, kl are grpo_score_fwd_kl's outputs. bf16 only. */
+ * reference). logp, lse, lse_ref, kl are grpo_score_fwd_kl's outputs. bf16 only. Workspace:
+ * grpo_workspace_bytes_kl. */
 int grpo_loss_bwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
                      int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
                      int32_t T, int32_t d, int32_t V, const float* logp, const float* lse,

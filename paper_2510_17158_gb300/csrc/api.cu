@@ -115,7 +115,10 @@ struct Layout {
   size_t fixed_end;     // end of the regions that do not depend on the vocabulary chunk
 };
 
-Layout make_layout(int S, int T, int d, int V, int dtype) {
+// `kl`: the exact-KL entry points' layout, with the reference model's packed hidden states and
+// forward statistics; the other entry points leave those two regions out (10 GB at 2 x 16
+// completions of T = 16384, d = 5120, V = 151936).
+Layout make_layout(int S, int T, int d, int V, int dtype, bool kl = false) {
   Layout L{};
   const size_t P = static_cast<size_t>(S) * T;
   L.rows_cap = static_cast<long long>((P + kTileRows - 1) / kTileRows) * kTileRows;
@@ -133,14 +136,14 @@ Layout make_layout(int S, int T, int d, int V, int dtype) {
   L.partials = off;
   if (bf16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
   L.partials2 = off;      // exact-KL forward only
-  if (bf16) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
+  if (bf16 && kl) off = align256(off + sizeof(float4) * L.num_strips * L.rows_cap);
   L.g = off;              off = align256(off + sizeof(float) * P);
   L.cvec = off;           off = align256(off + sizeof(float) * P);
   L.seq_loss = off;       off = align256(off + sizeof(float) * S);
   L.hp = off;             // packed hidden states (bf16 path)
   if (bf16) off = align256(off + static_cast<size_t>(L.rows_cap) * d * 2);
   L.hrp = off;            // packed reference hidden states (exact-KL path)
-  if (bf16) off = align256(off + static_cast<size_t>(L.rows_cap) * d * 2);
+  if (bf16 && kl) off = align256(off + static_cast<size_t>(L.rows_cap) * d * 2);
   L.fixed_end = off;
   return L;
 }
@@ -302,10 +305,14 @@ const char* grpo_kernel_name(int32_t kernel_id) {
   return kKernelNames[kernel_id];
 }
 
-size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
-                            int32_t vocab_chunk) {
+}  // extern "C"
+
+namespace {
+size_t workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                       int32_t vocab_chunk, bool kl) {
   if (!shape_ok(S, T, d, V) || check_dtype_shape(dtype, d) == GRPO_ERR_INVALID_ARG) return 0;
-  const Layout L = make_layout(S, T, d, V, dtype);
+  if (kl && dtype != GRPO_BF16) return 0;
+  const Layout L = make_layout(S, T, d, V, dtype, kl);
   if (dtype != GRPO_BF16) return L.fixed_end;
   int vc = L.v_round;
   if (vocab_chunk > 0) {
@@ -313,6 +320,19 @@ size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t 
     if (vc > L.v_round) vc = L.v_round;
   }
   return L.fixed_end + chunk_bytes(L, d, vc);
+}
+}  // namespace
+
+extern "C" {
+
+size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                            int32_t vocab_chunk) {
+  return workspace_bytes(S, T, d, V, dtype, vocab_chunk, false);
+}
+
+size_t grpo_workspace_bytes_kl(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
+                               int32_t vocab_chunk) {
+  return workspace_bytes(S, T, d, V, dtype, vocab_chunk, true);
 }
 
 int grpo_workspace_init(void* workspace, size_t workspace_bytes, grpo_stream_t stream) {
@@ -420,7 +440,7 @@ int loss_bwd_impl(int mode, const void* H, const void* W, int32_t dtype, const i
   if (!(eps_low >= 0.f) || !(eps_high >= 0.f) || !(beta >= 0.f) || !(norm >= 0.0))
     return GRPO_ERR_INVALID_ARG;
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
-  const Layout L = make_layout(S, T, d, V, dtype);
+  const Layout L = make_layout(S, T, d, V, dtype, mode == 2);
   if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);
@@ -582,7 +602,7 @@ int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const voi
   if (!aligned16(H) || !aligned16(W) || !aligned16(H_ref) || !aligned16(W_ref))
     return GRPO_ERR_INVALID_ARG;
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return GRPO_ERR_WORKSPACE;
-  const Layout L = make_layout(S, T, d, V, dtype);
+  const Layout L = make_layout(S, T, d, V, dtype, true);
   if (workspace_bytes < L.fixed_end) return GRPO_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const Views v = views(workspace, L);

@@ -48,6 +48,7 @@ _p, _i32, _i64, _f32, _f64, _sz = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int
 def _declare(lib):
     sig = {
         "grpo_workspace_bytes": (_sz, [_i32, _i32, _i32, _i32, _i32, _i32]),
+        "grpo_workspace_bytes_kl": (_sz, [_i32, _i32, _i32, _i32, _i32, _i32]),
         "grpo_workspace_init": (ctypes.c_int, [_p, _sz, _p]),
         "group_advantages": (ctypes.c_int, [_p, _p, _i32, _i32, _i32, _f32, _p, _p, _sz, _p]),
         "grpo_score_fwd": (ctypes.c_int, [_p, _p, _i32, _p, _p, _i32, _i32, _i32, _i32, _p, _p,
@@ -152,6 +153,12 @@ def grpo_workspace_bytes(S: int, T: int, d: int, V: int, dtype, vocab_chunk: int
     return int(_lib().grpo_workspace_bytes(S, T, d, V, code, vocab_chunk))
 
 
+def grpo_workspace_bytes_kl(S: int, T: int, d: int, V: int, dtype, vocab_chunk: int = 0) -> int:
+    """Workspace of the exact-KL entry points (also serves every other entry point)."""
+    code = dtype if isinstance(dtype, int) else (GRPO_BF16 if dtype == torch.bfloat16 else GRPO_F32)
+    return int(_lib().grpo_workspace_bytes_kl(S, T, d, V, code, vocab_chunk))
+
+
 @dataclass
 class Workspace:
     """A device workspace (torch-owned bytes) plus its size; initialised on creation."""
@@ -169,8 +176,11 @@ class Workspace:
         return ws
 
     @classmethod
-    def for_problem(cls, S, T, d, V, dtype, vocab_chunk=0, device="cuda") -> "Workspace":
-        n = grpo_workspace_bytes(S, T, d, V, dtype, vocab_chunk)
+    def for_problem(cls, S, T, d, V, dtype, vocab_chunk=0, device="cuda",
+                    kl=False) -> "Workspace":
+        """Workspace for this shape; `kl=True` sizes it for the exact-KL entry points."""
+        n = (grpo_workspace_bytes_kl if kl else grpo_workspace_bytes)(S, T, d, V, dtype,
+                                                                      vocab_chunk)
         if n == 0:
             raise ValueError("invalid problem shape")
         return cls.create(n, device)

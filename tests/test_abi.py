@@ -35,6 +35,13 @@ def test_workspace_bytes(lib):
     small = G.grpo_workspace_bytes(S, T, d, V, G.GRPO_BF16, 8192)
     assert small < full and small >= rows * 8192 * 2 + rows * d * 4
     assert G.grpo_workspace_bytes(0, T, d, V, G.GRPO_BF16, 0) == 0
+    # the exact-KL entry points add the reference model's packed rows (bf16) and its forward
+    # statistics (one float4 per 256 vocabulary columns), each over the packed-row capacity
+    rows = -(-S * T // 128) * 128
+    extra = G.grpo_workspace_bytes_kl(S, T, d, V, G.GRPO_BF16, 0) - full
+    want = rows * d * 2 + rows * 16 * -(-V // 256)
+    assert want <= extra <= want + 2 * 256
+    assert G.grpo_workspace_bytes_kl(4, 64, 64, 512, G.GRPO_F32, 0) == 0   # bf16 only
     assert G.grpo_workspace_bytes(4, 64, 64, 512, G.GRPO_F32, 0) > 0
 
 
