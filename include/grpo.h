@@ -60,10 +60,12 @@ typedef enum { GRPO_AGG_SEQ_MEAN = 0, GRPO_AGG_TOKEN_MEAN = 1 } grpo_agg;
 /* Bytes of workspace needed for a problem of this shape. `vocab_chunk` is how many vocabulary
  * columns of dL/dz the backward keeps at once (rounded up to a multiple of 256); 0 = the whole
  * vocabulary in one chunk (fastest; S*ceil(T/128)*128*V*2 bytes of scratch). Returns 0 for
- * invalid shapes. The workspace must be 256-byte aligned. The exact-KL entry points
- * (grpo_score_fwd_kl, grpo_loss_bwd_kl) need grpo_workspace_bytes_kl instead, which adds the
- * reference model's packed hidden states and forward statistics (bf16 only; 0 for f32); a
- * workspace of that size serves every entry point. */
+ * invalid shapes. The workspace must be 256-byte aligned. With less than this, the backward
+ * takes the widest vocabulary chunk that fits next to an f32 dH accumulator, and returns
+ * GRPO_ERR_WORKSPACE only if not even the fixed regions and one 256-column chunk fit. The
+ * exact-KL entry points (grpo_score_fwd_kl, grpo_loss_bwd_kl) also hold the reference model's
+ * packed hidden states and forward statistics: grpo_workspace_bytes_kl gives their size for the
+ * same chunking (bf16 only; 0 for f32), and a workspace of that size serves every entry point. */
 size_t grpo_workspace_bytes(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
                             int32_t vocab_chunk);
 size_t grpo_workspace_bytes_kl(int32_t S, int32_t T, int32_t d, int32_t V, int32_t dtype,
@@ -174,7 +176,7 @@ int grpo_rewards(const uint8_t* correct, const float* t_base, const float* t_new
  * grpo_score_fwd_kl computes grpo_score_fwd's outputs plus lse_ref [S,T] and kl [S,T] (0 at
  * unscored positions); both products stream through one tensor-core tile per 128 x 256 block,
  * the logits of neither model reach memory. H_ref [S,T,d], W_ref [V,d] bf16. Workspace:
- * grpo_workspace_bytes_kl (a smaller one returns GRPO_ERR_WORKSPACE). */
+ * grpo_workspace_bytes_kl. */
 int grpo_score_fwd_kl(const void* H, const void* W, const void* H_ref, const void* W_ref,
                       int32_t dtype, const int32_t* tokens, const uint8_t* mask, int32_t S,
                       int32_t T, int32_t d, int32_t V, float* logp, float* lse, float* entropy,

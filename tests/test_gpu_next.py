@@ -93,11 +93,6 @@ def test_exact_kl_parity(name, over):
     Hr, Wr = reference_model_inputs(b)
     H, W, tok, mask = (t.cuda() for t in (b.H, b.W, b.tokens, b.mask))
     S, T, d = H.shape
-    # the plain workspace lacks the reference model's regions: refused before any launch
-    with pytest.raises(G.GrpoError) as err:
-        G.grpo_score_fwd_kl(H, W, Hr.cuda(), Wr.cuda(), tok, mask,
-                            G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype))
-    assert err.value.status == -4    # GRPO_ERR_WORKSPACE
     ws = G.Workspace.for_problem(S, T, d, W.shape[0], H.dtype, kl=True)
     old, _ = oracle_inputs(b, old_scale=2.0)
     adv = G.group_advantages(b.rewards.cuda(), b.group_offsets.cuda(), ws)
